@@ -1,0 +1,115 @@
+/*
+ * sq_oracle.h -- CPU oracle for the SpecQuant draft/verify hot path.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only the test suite, the package's smoke check
+ * and the benchmark's CPU-baseline leg may load this code.  The GPU product
+ * path never calls it, links it or falls back to it.  It shares no header,
+ * helper, table or constant with the CUDA library: every definition below is
+ * written out from the paper and from the number-format standards it leans on.
+ *
+ * Paper: "SpecQuant -- Speculative Decoding with Multi-Parent Quantization
+ * for Adaptive LLM Inference".  Section references are to that paper:
+ *   Sec. III-A.1  low-precision parent  Q4  = f(W16, 4)
+ *   Sec. III-A.2  medium-precision parent Q8 = f(W16, 8)
+ *   Sec. III-A.3  full-precision parent Q16 = W16, and the token rule
+ *                 y_t = y_t^draft if the parent agrees, else f(x_{1:t-1})
+ *   Sec. III-D.2  draft generation, Sec. III-D.3 parent verification,
+ *   Sec. III-D.4  token acceptance or correction
+ *   Sec. I / II-A adherence to standard speculative decoding
+ *
+ * The paper fixes neither the quantisation scheme nor the sampling rule.
+ * The readings implemented here (symmetric INT4 with group 128 along K and
+ * fp16 scales, FP8-E4M3 with one fp32 scale per output row, the lossless
+ * speculative-sampling accept rule with a 2^-44 fixed-point CDF) are listed
+ * next to each function.
+ *
+ * Parity pins: every function here is checked by tests against something
+ * other than itself (library casts, brute force, exact rational arithmetic,
+ * exhaustive enumeration of the accept rule over the uniform grid).
+ */
+#ifndef SQ_ORACLE_H
+#define SQ_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes returned by the oracle (its own numbering). */
+#define OQ_OK 0
+#define OQ_BAD_ARG 1     /* shape not allowed, non-finite weight, ... */
+#define OQ_BAD_SEQ 2     /* at least one sequence was invalid (see oq_accept) */
+
+/* ---- number formats ------------------------------------------------------ */
+
+/* IEEE 754 binary16: bits -> exact value. */
+double oq_f16_decode(uint16_t h);
+/* Nearest binary16 to x, ties to the even bit pattern, overflow to +-inf. */
+uint16_t oq_f16_encode(double x);
+/* OCP FP8 E4M3 (bias 7, no infinities, S.1111.111 = NaN): bits -> value. */
+double oq_e4m3_decode(uint8_t c);
+/* Nearest E4M3 to x, ties to even mantissa, finite overflow saturates to
+ * +-448 ("satfinite"), sign of zero kept, NaN -> 0x7F. */
+uint8_t oq_e4m3_encode(double x);
+
+void oq_f16_decode_array(const uint16_t* h, int64_t n, double* out);
+void oq_f16_encode_array(const double* x, int64_t n, uint16_t* out);
+void oq_e4m3_encode_array(const float* x, int64_t n, uint8_t* out);
+
+/* ---- Sec. III-A.1: Q4 = f(W16, 4) ---------------------------------------- */
+/* w16 [N,K] fp16 row-major -> codes [N,K/2] (low nibble = even k, value
+ * c+8), scales [N,K/128] fp16 bits.  K % 128 == 0. */
+int oq_quantize_int4(const uint16_t* w16, int64_t N, int64_t K,
+                     uint8_t* codes, uint16_t* scales);
+/* codes/scales -> exact dequantised weights c*s as double [N,K]. */
+int oq_dequant_int4(const uint8_t* codes, const uint16_t* scales,
+                    int64_t N, int64_t K, double* w);
+
+/* ---- Sec. III-A.2: Q8 = f(W16, 8) ---------------------------------------- */
+/* w16 [N,K] -> codes [N,K] E4M3 bits, scales [N] fp32 (amax_n / 448). */
+int oq_quantize_fp8(const uint16_t* w16, int64_t N, int64_t K,
+                    uint8_t* codes, float* scales);
+int oq_dequant_fp8(const uint8_t* codes, const float* scales,
+                   int64_t N, int64_t K, double* w);
+
+/* ---- Sec. III-D.2/3: the linear layers of draft and verify passes -------- */
+/* y[M,N] = x[M,K] . w[N,K]^T (+ bias[N]), every product and sum in fp64. */
+void oq_linear(const double* x, const double* w, const double* bias,
+               int64_t M, int64_t N, int64_t K, double* y);
+/* h = silu(g) * u elementwise, silu(g) = g / (1 + exp(-g)), fp64. */
+void oq_silu_gate(const double* g, const double* u, int64_t n, double* h);
+
+/* ---- Sec. III-A.3 token rule and Sec. III-D.4 acceptance ------------------ */
+#define OQ_ACCEPT_SAMPLE 0
+#define OQ_ACCEPT_GREEDY 1
+/* floor(r * 2^44) for a finite r in [0, 1]. */
+uint64_t oq_fix44(float r);
+/* floor(u * S) for u in [0, 1), computed exactly. */
+uint64_t oq_scale_floor(float u, uint64_t S);
+/* p [B,K+1,V], q [B,K,V] (may be NULL when K == 0), draft [B,K],
+ * u [B,K+1] -> n_accepted [B], tokens [B,K+1] (-1 padded).
+ * A sequence whose draft token is outside [0,V), whose last uniform is
+ * outside [0,1), or whose resampling row has zero fixed-point mass gets
+ * n_accepted = -1 and all tokens -1; the call then returns OQ_BAD_SEQ. */
+int oq_accept(const float* p, const float* q, const int32_t* draft,
+              const float* u, int64_t B, int64_t K, int64_t V, int mode,
+              int32_t* n_accepted, int32_t* tokens);
+/* Draft-side sampling: token[b] ~ probs[b,:] by the same fixed-point
+ * inverse CDF (the K = 0 case of oq_accept in sampling mode). */
+int oq_sample(const float* probs, const float* u, int64_t B, int64_t V,
+              int32_t* tokens);
+
+/* ---- exhaustive-enumeration harness (sq_enumerate.c) --------------------- */
+/* Runs oq_accept on one sequence 2^grid_bits times, with the uniform at
+ * position `pos` set to m * 2^-grid_bits for every m, the others taken from
+ * u_fixed, and histograms the outcome: hist[n * V + token_at_n] counts,
+ * hist[(K+1)*V] counts invalid outcomes. */
+int oq_enum_sweep(const float* p, const float* q, const int32_t* draft,
+                  const float* u_fixed, int64_t K, int64_t V, int mode,
+                  int pos, int grid_bits, uint64_t* hist);
+
+#ifdef __cplusplus
+}
+#endif
+#endif
