@@ -1,0 +1,195 @@
+/*
+ * specquant.h -- C ABI of the GB300 (sm_103a) SpecQuant draft/verify hot path.
+ *
+ * Paper: "SpecQuant -- Speculative Decoding with Multi-Parent Quantization
+ * for Adaptive LLM Inference".  One FP16 parent W16 gives an INT4 variant
+ * Q4 = f(W16, 4) (Sec. III-A.1) and an FP8 variant Q8 = f(W16, 8)
+ * (Sec. III-A.2).  The variants draft tokens (Sec. III-D.2), the parent
+ * verifies the draft block in one pass (Sec. III-D.3), and the accept step
+ * keeps the agreeing prefix and supplies the correction (Sec. III-A.3 token
+ * rule, Sec. III-D.4).
+ *
+ * Conventions shared by every call
+ *  - Every tensor pointer is a DEVICE pointer owned by the caller; the
+ *    library allocates nothing in these calls and keeps no reference after
+ *    the call returns.  Row-major, densely packed, no strides.
+ *  - Every call is asynchronous and ordered on `stream` (NULL = the legacy
+ *    default stream).  Kernels are launched with programmatic dependent
+ *    launch allowed, so a call may start fetching its weights while the
+ *    previous kernel on the stream finishes; it reads activations and writes
+ *    outputs only after that kernel completed.
+ *  - Return value: SQ_OK, or an error code whose text sq_last_error()
+ *    returns (per host thread).  Arguments are validated on the host before
+ *    anything is launched; an invalid call launches nothing.  No call traps,
+ *    aborts or throws.
+ *  - Data-dependent problems found on the device (a non-finite weight, a
+ *    draft token outside [0, V), a resampling row without mass) set bits of
+ *    a per-device status word that sq_check() reads and clears.
+ *  - fp16 means IEEE binary16; E4M3 means the OCP FP8 E4M3 format.
+ */
+#ifndef SPECQUANT_H
+#define SPECQUANT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A CUDA runtime stream (cudaStream_t); declared here so that callers need
+ * no CUDA header. */
+typedef struct CUstream_st* sq_stream_t;
+
+typedef enum {
+  SQ_OK = 0,
+  SQ_ERR_INVALID_ARG = 1,  /* NULL pointer, negative size, unknown enum   */
+  SQ_ERR_SHAPE = 2,        /* sizes outside the documented limits         */
+  SQ_ERR_ALIGN = 3,        /* pointer not 16-byte aligned where required  */
+  SQ_ERR_UNSUPPORTED = 4,  /* valid request this build does not implement */
+  SQ_ERR_WORKSPACE = 5,    /* workspace NULL or smaller than required     */
+  SQ_ERR_CUDA = 6,         /* a CUDA runtime call failed (message says)   */
+  SQ_ERR_DEVICE = 7        /* sq_check: the device flagged invalid data   */
+} sq_status;
+
+typedef enum { SQ_INT4_G128 = 1, SQ_FP8_E4M3_ROW = 2 } sq_qkind;
+typedef enum { SQ_ACCEPT_SAMPLE = 0, SQ_ACCEPT_GREEDY = 1 } sq_accept_mode;
+
+/* Device status bits reported through sq_check(). */
+#define SQ_DEV_NONFINITE_WEIGHT 0x1u  /* sq_quantize saw a NaN or infinity  */
+#define SQ_DEV_BAD_DRAFT_TOKEN  0x2u  /* sq_accept: draft token not in [0,V) */
+#define SQ_DEV_NO_MASS          0x4u  /* sq_accept/sq_sample: row w/o mass   */
+#define SQ_DEV_BAD_UNIFORM      0x8u  /* resampling uniform not in [0,1)     */
+
+/* Thread-local text of the last error raised on this host thread. */
+const char* sq_last_error(void);
+/* Fixed name of a status code. */
+const char* sq_status_string(sq_status s);
+/* Library version, major * 10000 + minor * 100 + patch. */
+int sq_version(void);
+
+/* Synchronises `stream`, then reads and clears the device status word of
+ * the current device.  Returns SQ_OK, SQ_ERR_DEVICE (bits in *device_bits,
+ * which may be NULL) or SQ_ERR_CUDA. */
+sq_status sq_check(sq_stream_t stream, uint32_t* device_bits);
+
+/* ------------------------------------------------------------------------
+ * Sec. III-A.1 / III-A.2: derive the draft variants from the FP16 parent.
+ *
+ * sq_quantized_bytes: bytes of the code and scale buffers of a variant of
+ * an [N, K] weight (scale_bytes may be NULL); 0 for an invalid request.
+ *
+ * sq_quantize: w16 fp16 [N, K] -> codes + scales.
+ *   SQ_INT4_G128 (the paper fixes no scheme; this is symmetric RTN INT4):
+ *     per row n and 128-wide group g along K: amax = max|w|,
+ *     s = fp16(fp32(amax / 7)), s = 2^-24 if amax > 0 rounded s to zero,
+ *     c = clamp(rint(fp32(w / s)), -8, 7) (ties to even), c = 0 if s = 0.
+ *     codes: uint8 [N, K/2], byte j of a row holds k = 2j in its low nibble
+ *     and k = 2j+1 in its high nibble, each as c + 8.
+ *     scales: fp16 [N, K/128].  Requires K % 128 == 0.
+ *   SQ_FP8_E4M3_ROW: s_n = fp32(amax_n / 448) (fp32 [N]),
+ *     code = E4M3(fp32(w / s_n)) rounded to nearest even, saturating to
+ *     +-448; code +0 for a row with s_n = 0.  codes: uint8 [N, K].
+ *     Requires K % 16 == 0.
+ *   Codes and scales are bit-identical to the definition above.  Alignment:
+ *   w16, codes 16 B.  A non-finite weight sets SQ_DEV_NONFINITE_WEIGHT.
+ * ---------------------------------------------------------------------- */
+size_t sq_quantized_bytes(sq_qkind kind, int64_t N, int64_t K, size_t* scale_bytes);
+sq_status sq_quantize(const void* w16, int64_t N, int64_t K, sq_qkind kind,
+                      void* codes, void* scales, sq_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Sec. III-D.2 (draft pass) / III-D.3 (verify pass): linear layers.
+ *
+ *   y[m, n] = sum_k x[m, k] * w'[n, k] (+ bias[n]),  m < M, n < N,
+ * with w' the dequantised weight: c * s (INT4), s_n * E4M3(c) (FP8) or the
+ * fp16 parent weight (sq_verify).  x: fp16 [M, K]; y: fp16 [M, N]; bias:
+ * fp16 [N] or NULL.  Products are exact and sums are fp32; y is rounded to
+ * nearest fp16 once.  1 <= M <= 256; N >= 1; K as for sq_quantize (INT4:
+ * K % 128 == 0, FP8: K % 16 == 0, FP16: K % 8 == 0).  x, codes, w16 and y
+ * must be 16-byte aligned.  M < 16 runs on CUDA cores (GEMV family); larger
+ * M runs on the tcgen05 tensor-core tile path where this build has it.
+ * y must not overlap x, the weights or the scales.
+ * ---------------------------------------------------------------------- */
+sq_status sq_linear_w4a16(const void* x, const void* codes, const void* scales,
+                          const void* bias, void* y, int M, int64_t N, int64_t K,
+                          sq_stream_t stream);
+sq_status sq_linear_fp8(const void* x, const void* codes, const float* scales,
+                        const void* bias, void* y, int M, int64_t N, int64_t K,
+                        sq_stream_t stream);
+sq_status sq_verify(const void* x, const void* w16, const void* bias, void* y,
+                    int M, int64_t N, int64_t K, sq_stream_t stream);
+
+/* Fused epilogues of the same three linear layers (the transformer block's
+ * MLP, not specified by the paper).
+ *  SQ_EPI_SILU_GATE: the weight holds 2N rows, rows [0, N) the gate and
+ *    rows [N, 2N) the up projection; y[m, n] = silu(g) * u with
+ *    g = x . w'[n], u = x . w'[N + n], silu(g) = g / (1 + exp(-g)), in fp32.
+ *    bias (if any) has 2N entries.
+ *  SQ_EPI_RESIDUAL: y[m, n] = residual[m, n] + x . w'[n] (+ bias[n]);
+ *    residual fp16 [M, N]; it may be the same buffer as y (in place). */
+typedef enum { SQ_EPI_NONE = 0, SQ_EPI_SILU_GATE = 1, SQ_EPI_RESIDUAL = 2 } sq_epilogue;
+typedef enum { SQ_W_FP16 = 0, SQ_W_INT4 = 1, SQ_W_FP8 = 2 } sq_wkind;
+
+/* Generic form of the three linear calls: wkind selects the weight format
+ * (w = w16 for SQ_W_FP16, codes otherwise; scales NULL for SQ_W_FP16),
+ * epi the epilogue.  residual is read only for SQ_EPI_RESIDUAL. */
+sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void* scales,
+                       const void* bias, const void* residual, sq_epilogue epi, void* y,
+                       int M, int64_t N, int64_t K, sq_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Sec. III-A.3 token rule and Sec. III-D.4 acceptance / correction, for a
+ * batch of B independent sequences with K draft tokens each over a
+ * vocabulary of V tokens.
+ *
+ *   p      fp32 [B, K+1, V]  target (parent) probabilities, positions 0..K
+ *   q      fp32 [B, K, V]    draft probabilities (NULL allowed when K == 0
+ *                            or mode == SQ_ACCEPT_GREEDY)
+ *   draft  int32 [B, K]      draft tokens
+ *   u      fp32 [B, K+1]     uniforms in [0, 1): u[b, i] for the test of
+ *                            draft i, u[b, K] for the correction/bonus draw
+ *   n_accepted int32 [B], tokens int32 [B, K+1] (outputs)
+ *
+ * SQ_ACCEPT_SAMPLE (the lossless speculative-sampling rule the paper says
+ * it follows, Sec. I): draft i is kept iff u_i * q_i(x_i) < p_i(x_i),
+ * evaluated exactly; n = number kept before the first rejection.  The
+ * correction token is drawn from r = max(0, p_n - q_n) (fp32 subtraction)
+ * if n < K, else from r = p_K; if n < K and r has no mass, from p_n.  The
+ * draw is a fixed-point inverse CDF: R_v = floor(r_v * 2^44),
+ * S = sum_v R_v, T = floor(u_K * S), token = min{v : R_0 + .. + R_v > T};
+ * every integer sum is exact, so the result does not depend on reduction
+ * order and is bit-identical to the definition.
+ * SQ_ACCEPT_GREEDY (the token rule read literally): draft i is kept iff it
+ * equals argmax p_i (lowest index on ties); the correction is argmax p_n.
+ *
+ * tokens[b] = draft[b, 0..n-1], correction, then -1 up to K+1 entries;
+ * n_accepted[b] = n.  A sequence with a draft token outside [0, V), a
+ * correction uniform outside [0, 1) or a correction row without mass gets
+ * n_accepted = -1 and all tokens -1, and sets the matching device status bit.
+ *
+ * Limits: B >= 0, 0 <= K <= 16, 1 <= V < 2^20.  p, q in [0, 1], finite
+ * (rows need not sum to exactly 1).  Pointers 4-byte aligned (16 B for p
+ * and q when V % 4 == 0 lets the kernel use vector loads).
+ *
+ * workspace: device memory of at least sq_accept_workspace_bytes(B, K, V)
+ * bytes, 16-byte aligned.  It must be zero-filled before its first use; each
+ * call leaves it zero-filled when it completes.  Calls that share one
+ * workspace must not run concurrently on the GPU.
+ * ---------------------------------------------------------------------- */
+size_t sq_accept_workspace_bytes(int B, int K, int64_t V);
+sq_status sq_accept(const float* p, const float* q, const int32_t* draft, const float* u,
+                    int B, int K, int64_t V, sq_accept_mode mode,
+                    int32_t* n_accepted, int32_t* tokens,
+                    void* workspace, size_t ws_bytes, sq_stream_t stream);
+
+/* Draft-side sampling, token[b] ~ probs[b, :] with uniform u[b]: the K = 0
+ * case of sq_accept in sampling mode (same fixed-point inverse CDF, same
+ * workspace rules, workspace size sq_accept_workspace_bytes(B, 0, V)). */
+sq_status sq_sample(const float* probs, const float* u, int B, int64_t V, int32_t* tokens,
+                    void* workspace, size_t ws_bytes, sq_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

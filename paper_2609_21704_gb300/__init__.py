@@ -1,0 +1,185 @@
+"""GB300-native (sm_103a) SpecQuant draft/verify hot path.
+
+A thin ctypes binding over ``libspecquant.so`` (the C ABI declared in
+``include/specquant.h``).  Functions keep the C names and only marshal
+arguments: torch tensors supply device memory (``data_ptr()``) and sizes,
+``torch.cuda`` supplies the stream.  Every step of the path runs in the
+library's CUDA kernels; there is no CPU fallback, and importing a function
+fails loudly when the library has not been built.
+
+Paper: "SpecQuant -- Speculative Decoding with Multi-Parent Quantization for
+Adaptive LLM Inference" (Sec. III-A variants, Sec. III-D pipeline).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from ._build import LIB as LIB_PATH
+from ._build import build
+
+__all__ = [
+    "SQError", "build", "load", "LIB_PATH",
+    "SQ_INT4_G128", "SQ_FP8_E4M3_ROW", "SQ_ACCEPT_SAMPLE", "SQ_ACCEPT_GREEDY",
+    "SQ_EPI_NONE", "SQ_EPI_SILU_GATE", "SQ_EPI_RESIDUAL", "SQ_W_FP16", "SQ_W_INT4", "SQ_W_FP8",
+    "sq_quantized_bytes", "sq_quantize", "sq_linear_w4a16", "sq_linear_fp8", "sq_verify",
+    "sq_linear_ex", "sq_accept_workspace_bytes", "sq_accept", "sq_sample", "sq_check",
+    "sq_version", "EXPORTED_SYMBOLS",
+]
+
+SQ_OK = 0
+SQ_INT4_G128, SQ_FP8_E4M3_ROW = 1, 2
+SQ_ACCEPT_SAMPLE, SQ_ACCEPT_GREEDY = 0, 1
+SQ_EPI_NONE, SQ_EPI_SILU_GATE, SQ_EPI_RESIDUAL = 0, 1, 2
+SQ_W_FP16, SQ_W_INT4, SQ_W_FP8 = 0, 1, 2
+SQ_DEV_NONFINITE_WEIGHT, SQ_DEV_BAD_DRAFT_TOKEN, SQ_DEV_NO_MASS, SQ_DEV_BAD_UNIFORM = 1, 2, 4, 8
+
+_P = ctypes.c_void_p
+_I64 = ctypes.c_int64
+_INT = ctypes.c_int
+_SIZE = ctypes.c_size_t
+_SIGS = {
+    "sq_last_error": (ctypes.c_char_p, []),
+    "sq_status_string": (ctypes.c_char_p, [_INT]),
+    "sq_version": (_INT, []),
+    "sq_check": (_INT, [_P, ctypes.POINTER(ctypes.c_uint32)]),
+    "sq_quantized_bytes": (_SIZE, [_INT, _I64, _I64, ctypes.POINTER(_SIZE)]),
+    "sq_quantize": (_INT, [_P, _I64, _I64, _INT, _P, _P, _P]),
+    "sq_linear_w4a16": (_INT, [_P, _P, _P, _P, _P, _INT, _I64, _I64, _P]),
+    "sq_linear_fp8": (_INT, [_P, _P, _P, _P, _P, _INT, _I64, _I64, _P]),
+    "sq_verify": (_INT, [_P, _P, _P, _P, _INT, _I64, _I64, _P]),
+    "sq_linear_ex": (_INT, [_INT, _P, _P, _P, _P, _P, _INT, _P, _INT, _I64, _I64, _P]),
+    "sq_accept_workspace_bytes": (_SIZE, [_INT, _INT, _I64]),
+    "sq_accept": (_INT, [_P, _P, _P, _P, _INT, _INT, _I64, _INT, _P, _P, _P, _SIZE, _P]),
+    "sq_sample": (_INT, [_P, _P, _INT, _I64, _P, _P, _SIZE, _P]),
+}
+EXPORTED_SYMBOLS = tuple(_SIGS)
+
+_lib = None
+
+
+class SQError(RuntimeError):
+    """A call into libspecquant returned an error status."""
+
+    def __init__(self, fn: str, status: int, msg: str):
+        super().__init__(f"{fn}: {msg} (status {status})")
+        self.status = status
+
+
+def load(path: str | None = None) -> ctypes.CDLL:
+    """Load libspecquant.so (built by ``build()``); raises if it is missing."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise ImportError(f"{p} is not built; run paper_2609_21704_gb300.build() (needs nvcc)")
+    lib = ctypes.CDLL(p)
+    for name, (res, args) in _SIGS.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    if path is None:
+        _lib = lib
+    return lib
+
+
+def _check(fn: str, status: int) -> None:
+    if status != SQ_OK:
+        lib = load()
+        raise SQError(fn, status, lib.sq_last_error().decode(errors="replace"))
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("expected a torch.Tensor")
+    if not t.is_cuda:
+        raise ValueError("tensor must live on a CUDA device")
+    if not t.is_contiguous():
+        raise ValueError("tensor must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def sq_version() -> int:
+    return load().sq_version()
+
+
+def sq_quantized_bytes(kind: int, N: int, K: int):
+    sb = _SIZE(0)
+    cb = load().sq_quantized_bytes(kind, N, K, ctypes.byref(sb))
+    return int(cb), int(sb.value)
+
+
+def sq_quantize(w16, kind, codes, scales, stream=None) -> None:
+    N, K = w16.shape
+    _check("sq_quantize", load().sq_quantize(_ptr(w16), N, K, kind, _ptr(codes), _ptr(scales),
+                                             _stream(stream)))
+
+
+def sq_linear_ex(wkind, x, w, scales, bias, residual, epi, y, stream=None) -> None:
+    M, K = x.shape
+    N = y.shape[1]
+    _check("sq_linear_ex", load().sq_linear_ex(wkind, _ptr(x), _ptr(w), _ptr(scales), _ptr(bias),
+                                               _ptr(residual), epi, _ptr(y), M, N, K,
+                                               _stream(stream)))
+
+
+def sq_linear_w4a16(x, codes, scales, bias, y, stream=None) -> None:
+    M, K = x.shape
+    N = y.shape[1]
+    _check("sq_linear_w4a16", load().sq_linear_w4a16(_ptr(x), _ptr(codes), _ptr(scales), _ptr(bias),
+                                                     _ptr(y), M, N, K, _stream(stream)))
+
+
+def sq_linear_fp8(x, codes, scales, bias, y, stream=None) -> None:
+    M, K = x.shape
+    N = y.shape[1]
+    _check("sq_linear_fp8", load().sq_linear_fp8(_ptr(x), _ptr(codes), _ptr(scales), _ptr(bias),
+                                                 _ptr(y), M, N, K, _stream(stream)))
+
+
+def sq_verify(x, w16, bias, y, stream=None) -> None:
+    M, K = x.shape
+    N = y.shape[1]
+    _check("sq_verify", load().sq_verify(_ptr(x), _ptr(w16), _ptr(bias), _ptr(y), M, N, K,
+                                         _stream(stream)))
+
+
+def sq_accept_workspace_bytes(B: int, K: int, V: int) -> int:
+    return int(load().sq_accept_workspace_bytes(B, K, V))
+
+
+def sq_accept(p, q, draft, u, mode, n_accepted, tokens, workspace, stream=None) -> None:
+    B, K1, V = p.shape
+    _check("sq_accept", load().sq_accept(_ptr(p), _ptr(q), _ptr(draft), _ptr(u), B, K1 - 1, V, mode,
+                                         _ptr(n_accepted), _ptr(tokens), _ptr(workspace),
+                                         workspace.numel() * workspace.element_size(),
+                                         _stream(stream)))
+
+
+def sq_sample(probs, u, tokens, workspace, stream=None) -> None:
+    B, V = probs.shape
+    _check("sq_sample", load().sq_sample(_ptr(probs), _ptr(u), B, V, _ptr(tokens), _ptr(workspace),
+                                         workspace.numel() * workspace.element_size(),
+                                         _stream(stream)))
+
+
+def sq_check(stream=None) -> int:
+    """Synchronise the stream; return the device status bits (0 when clean)."""
+    bits = ctypes.c_uint32(0)
+    st = load().sq_check(_stream(stream), ctypes.byref(bits))
+    if st not in (SQ_OK, 7):
+        _check("sq_check", st)
+    return int(bits.value)

@@ -1,0 +1,311 @@
+// sq_accept.cu -- accept / reject / resample over the vocabulary.
+//
+// Sec. III-A.3 (token rule) and Sec. III-D.4 (token acceptance or
+// correction); sampling mode is the lossless speculative-sampling rule the
+// paper says it adheres to (Sec. I).  Semantics are stated in specquant.h.
+//
+// Layout of the work: one CTA per (sequence b, vocabulary chunk c) of 2048
+// entries.  Every CTA evaluates the K accept tests of its sequence (K
+// gathers), then reduces its chunk of the correction row to a 64-bit
+// fixed-point partial sum (sampling) or a packed (value, index) maximum per
+// position (greedy).  The partials go to the workspace; the last CTA of a
+// sequence to arrive (atomic ticket) combines them, turns the uniform into
+// an integer target T = floor(u * S), finds the chunk holding T and scans
+// that chunk alone for the token.  All sums are integer, so the outcome is
+// independent of the order in which CTAs arrive.
+//
+// Bytes per sequence: sampling 2 V fp32 (p_n and q_n) + 2K gathers;
+// greedy (K+1) V fp32.
+#include "sq_internal.h"
+
+namespace sq {
+
+__device__ unsigned int g_accept_status;
+
+// floor(r * 2^44) from the fp32 bits of r in [0, 1] (exact integer shifts).
+__device__ __forceinline__ unsigned long long fix44(float r) {
+  const uint32_t b = __float_as_uint(r);
+  const uint32_t e = (b >> 23) & 0xffu;
+  if ((b >> 31) || e == 0) return 0ull;  // zero, negative, or below 2^-126
+  const unsigned long long mant = (unsigned long long)((b & 0x7fffffu) | 0x800000u);
+  const int sh = (int)e - 150 + 44;      // r = mant * 2^(e-150)
+  if (sh >= 0) return mant << sh;
+  if (sh <= -64) return 0ull;
+  return mant >> (-sh);
+}
+
+// floor(u * S) for u in [0, 1), exact (128-bit product of the 24-bit
+// significand and S, then a right shift).
+__device__ __forceinline__ unsigned long long scale_floor(float u, unsigned long long S) {
+  const uint32_t b = __float_as_uint(u);
+  const uint32_t e = (b >> 23) & 0xffu;
+  if ((b >> 31) || e == 0 || S == 0) return 0ull;
+  const unsigned long long mant = (unsigned long long)((b & 0x7fffffu) | 0x800000u);
+  const int shift = 150 - (int)e;        // u = mant / 2^shift, shift >= 24
+  const unsigned long long lo = mant * S;
+  const unsigned long long hi = __umul64hi(mant, S);
+  if (shift >= 128) return 0ull;
+  if (shift >= 64) return hi >> (shift - 64);
+  return (lo >> shift) | (hi << (64 - shift));
+}
+
+__device__ __forceinline__ unsigned long long warp_sum_u64(unsigned long long v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ unsigned long long warp_max_u64(unsigned long long v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const unsigned long long w = __shfl_xor_sync(0xffffffffu, v, o);
+    v = w > v ? w : v;
+  }
+  return v;
+}
+
+// (value, index) -> key whose unsigned maximum is the largest value with
+// the lowest index (values are non-negative, so their bits order like ints).
+__device__ __forceinline__ unsigned long long argmax_key(float v, int64_t idx) {
+  return ((unsigned long long)__float_as_uint(v) << 32) | (0xffffffffull - (unsigned long long)idx);
+}
+
+constexpr int kAcceptThreads = 256;
+
+__global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ unsigned long long red[kAcceptThreads / 32][17];
+  __shared__ int s_n, s_valid, s_last;
+  __shared__ unsigned long long s_T;
+  __shared__ int s_chunk, s_use_p, s_token;
+
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t bc = blockIdx.x;
+  const int b = (int)(bc / a.C), c = (int)(bc - (int64_t)b * a.C);
+  const int K = a.K;
+  const int64_t V = a.V;
+  const float* pb = a.p + (int64_t)b * (K + 1) * V;
+  const float* qb = a.q ? a.q + (int64_t)b * K * V : nullptr;
+  const int32_t* xb = a.draft + (int64_t)b * K;
+  const float* ub = a.u + (int64_t)b * (K + 1);
+  const int64_t v0 = (int64_t)c * a.chunk;
+  const int64_t v1 = v0 + a.chunk < V ? v0 + a.chunk : V;
+  unsigned long long* part = a.part + ((int64_t)b * a.C + c) * a.slots;
+
+  // ---- validity and (sampling) the accept tests, evaluated by warp 0
+  if (warp == 0) {
+    bool bad = false, acc = true;
+    if (lane < K) {
+      const int32_t x = xb[lane];
+      bad = (x < 0 || (int64_t)x >= V);
+      if (!bad && a.mode == SQ_ACCEPT_SAMPLE)
+        acc = (double)ub[lane] * (double)qb[(int64_t)lane * V + x] < (double)pb[(int64_t)lane * V + x];
+    }
+    const float uk = ub[K];
+    const bool bad_u = !(uk >= 0.0f && uk < 1.0f);
+    const unsigned bad_mask = __ballot_sync(0xffffffffu, bad);
+    const unsigned rej_mask = __ballot_sync(0xffffffffu, lane < K && !acc);
+    if (lane == 0) {
+      s_valid = (bad_mask == 0u) && !bad_u;
+      s_n = rej_mask ? (__ffs(rej_mask) - 1) : K;
+      if (c == 0 && bad_mask) atomicOr(&g_accept_status, SQ_DEV_BAD_DRAFT_TOKEN);
+      if (c == 0 && bad_u) atomicOr(&g_accept_status, SQ_DEV_BAD_UNIFORM);
+    }
+  }
+  __syncthreads();
+  const int n = s_n;
+
+  // ---- chunk partials
+  if (a.mode == SQ_ACCEPT_SAMPLE) {
+    const float* pn = pb + (int64_t)n * V;
+    const float* qn = (n < K) ? qb + (int64_t)n * V : nullptr;
+    unsigned long long sr = 0, sp = 0;
+    for (int64_t v = v0 + tid; v < v1; v += kAcceptThreads) {
+      const float pv = pn[v];
+      if (qn) {
+        const float d = pv - qn[v];
+        sr += fix44(d > 0.0f ? d : 0.0f);
+        sp += fix44(pv);
+      } else {
+        sr += fix44(pv);
+      }
+    }
+    sr = warp_sum_u64(sr);
+    sp = warp_sum_u64(sp);
+    if (lane == 0) {
+      red[warp][0] = sr;
+      red[warp][1] = sp;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      unsigned long long tr = 0, tp = 0;
+      for (int w = 0; w < kAcceptThreads / 32; ++w) {
+        tr += red[w][0];
+        tp += red[w][1];
+      }
+      part[0] = tr;
+      part[1] = tp;
+    }
+  } else {
+    // greedy: per position i, the maximum key over the chunk
+    for (int i = 0; i <= K; ++i) {
+      const float* pi = pb + (int64_t)i * V;
+      unsigned long long best = 0;
+      for (int64_t v = v0 + tid; v < v1; v += kAcceptThreads) {
+        const unsigned long long k = argmax_key(pi[v], v);
+        best = k > best ? k : best;
+      }
+      best = warp_max_u64(best);
+      if (lane == 0) red[warp][i] = best;
+    }
+    __syncthreads();
+    if (tid <= K) {
+      unsigned long long best = 0;
+      for (int w = 0; w < kAcceptThreads / 32; ++w) best = red[w][tid] > best ? red[w][tid] : best;
+      part[tid] = best;
+    }
+  }
+
+  // ---- ticket: the last CTA of the sequence finishes it
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    const unsigned ticket = atomicAdd(&a.counter[b], 1u);
+    s_last = (ticket == (unsigned)(a.C - 1));
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const unsigned long long* pall = a.part + (int64_t)b * a.C * a.slots;
+  int32_t* tok = a.tok_out + (int64_t)b * (K + 1);
+
+  if (a.mode == SQ_ACCEPT_GREEDY) {
+    if (tid == 0) {
+      int nn = K;
+      int64_t am_n = -1;
+      for (int i = 0; i <= K; ++i) {
+        unsigned long long best = 0;
+        for (int cc = 0; cc < a.C; ++cc) {
+          const unsigned long long k = __ldcg(pall + (int64_t)cc * a.slots + i);
+          best = k > best ? k : best;
+        }
+        const int64_t am = (int64_t)(0xffffffffull - (best & 0xffffffffull));
+        if (i < nn && i < K && am != xb[i]) nn = i;
+        if (i == nn) {
+          am_n = am;
+          break;
+        }
+      }
+      const bool ok = s_valid != 0;
+      if (a.n_out) a.n_out[b] = ok ? nn : -1;
+      for (int i = 0; i <= K; ++i) tok[i] = ok ? (i < nn ? xb[i] : (i == nn ? (int32_t)am_n : -1)) : -1;
+      a.counter[b] = 0u;
+    }
+    return;
+  }
+
+  // sampling: pick the row, the total mass, the target and its chunk
+  if (tid == 0) {
+    unsigned long long S = 0;
+    for (int cc = 0; cc < a.C; ++cc) S += __ldcg(pall + (int64_t)cc * a.slots + 0);
+    int use_p = 0;
+    if (S == 0 && n < K) {
+      for (int cc = 0; cc < a.C; ++cc) S += __ldcg(pall + (int64_t)cc * a.slots + 1);
+      use_p = 1;
+    }
+    int ok = s_valid && S != 0;
+    if (s_valid && S == 0) atomicOr(&g_accept_status, SQ_DEV_NO_MASS);
+    const unsigned long long T = ok ? scale_floor(ub[K], S) : 0ull;
+    unsigned long long before = 0;
+    int cs = a.C - 1;
+    for (int cc = 0; cc < a.C; ++cc) {
+      const unsigned long long pc = __ldcg(pall + (int64_t)cc * a.slots + use_p);
+      if (before + pc > T) {
+        cs = cc;
+        break;
+      }
+      before += pc;
+    }
+    s_T = T - before;
+    s_chunk = cs;
+    s_use_p = use_p;
+    s_valid = ok;
+    s_token = -1;
+  }
+  __syncthreads();
+  if (s_valid) {
+    const float* pn = pb + (int64_t)n * V;
+    const float* qn = (n < K && !s_use_p) ? qb + (int64_t)n * V : nullptr;
+    const int64_t w0 = (int64_t)s_chunk * a.chunk;
+    const int64_t w1 = w0 + a.chunk < V ? w0 + a.chunk : V;
+    const unsigned long long T = s_T;
+    unsigned long long run = 0;  // mass of the sub-blocks already scanned
+    for (int64_t base = w0; base < w1; base += kAcceptThreads) {
+      const int64_t v = base + tid;
+      unsigned long long R = 0;
+      if (v < w1) {
+        const float pv = pn[v];
+        if (qn) {
+          const float d = pv - qn[v];
+          R = fix44(d > 0.0f ? d : 0.0f);
+        } else {
+          R = fix44(pv);
+        }
+      }
+      // inclusive block scan of R
+      unsigned long long incl = R;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += t;
+      }
+      if (lane == 31) red[warp][0] = incl;
+      __syncthreads();
+      unsigned long long wbase = 0, total = 0;
+      for (int w = 0; w < kAcceptThreads / 32; ++w) {
+        if (w < warp) wbase += red[w][0];
+        total += red[w][0];
+      }
+      incl += wbase + run;
+      const unsigned long long excl = incl - R;
+      if (excl <= T && incl > T) s_token = (int)v;  // exactly one thread matches
+      __syncthreads();
+      if (s_token >= 0) break;
+      run += total;
+    }
+  }
+  __syncthreads();
+  if (tid == 0) {
+    const bool ok = s_valid && s_token >= 0;
+    if (a.n_out) a.n_out[b] = ok ? n : -1;
+    for (int i = 0; i <= K; ++i) tok[i] = ok ? (i < n ? xb[i] : (i == n ? s_token : -1)) : -1;
+    a.counter[b] = 0u;
+  }
+}
+
+size_t accept_workspace_bytes(int B, int K, int64_t V) {
+  if (B < 0 || K < 0 || V <= 0) return 0;
+  const int64_t C = (V + kAcceptChunk - 1) / kAcceptChunk;
+  const int64_t slots = K + 1 > 2 ? K + 1 : 2;
+  const size_t part = (size_t)B * (size_t)C * (size_t)slots * 8u;
+  const size_t ctr = (((size_t)B * 4u) + 15u) & ~(size_t)15u;
+  return ctr + part + 16u;
+}
+
+cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t st) {
+  if (a.B == 0) return cudaSuccess;
+  const int64_t blocks = (int64_t)a.B * a.C;
+  return launch_pdl(accept_kernel, dim3((unsigned)blocks), dim3(kAcceptThreads), 0, st, a);
+}
+
+cudaError_t take_accept_status(uint32_t* bits) {
+  uint32_t v = 0, zero = 0;
+  cudaError_t e = cudaMemcpyFromSymbol(&v, g_accept_status, sizeof(v));
+  if (e != cudaSuccess) return e;
+  if (v) e = cudaMemcpyToSymbol(g_accept_status, &zero, sizeof(zero));
+  *bits |= v;
+  return e;
+}
+
+}  // namespace sq

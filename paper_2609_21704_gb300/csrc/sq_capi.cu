@@ -1,0 +1,328 @@
+// sq_capi.cu -- the C ABI (include/specquant.h): argument validation, status
+// reporting and dispatch to the kernels.  Nothing here computes any part of
+// the hot path; it only checks arguments and launches.
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <string>
+
+#include "sq_internal.h"
+
+namespace sq {
+
+static thread_local std::string g_last_error;
+
+static sq_status fail(sq_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+static sq_status cuda_fail(cudaError_t e, const char* where) {
+  return fail(SQ_ERR_CUDA, "%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+static bool aligned(const void* p, uintptr_t a) { return ((uintptr_t)p % a) == 0; }
+
+int device_sm_count() {
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return kNumSMs;
+  if (cache[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = kNumSMs;
+    cache[dev] = n;
+  }
+  return cache[dev];
+}
+
+static int device_max_smem() {
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 227 * 1024;
+  if (cache[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+        n <= 0)
+      n = 227 * 1024;
+    cache[dev] = n;
+  }
+  return cache[dev];
+}
+
+// ---------------------------------------------------------------- GEMV plan
+
+static int sub_of(int wk) { return wk == SQ_W_INT4 ? 4 : wk == SQ_W_FP8 ? 2 : 1; }
+static int64_t weights_per_piece(int wk) { return wk == SQ_W_INT4 ? 32 : wk == SQ_W_FP8 ? 16 : 8; }
+static int64_t row_bytes_of(int wk, int64_t K) {
+  return wk == SQ_W_INT4 ? K / 2 : wk == SQ_W_FP8 ? K : 2 * K;
+}
+
+size_t gemv_smem_bytes(int wk, int mr, int64_t K) {
+  const int64_t pieces = K / weights_per_piece(wk);
+  const int64_t ppad = (pieces + 31) / 32 * 32;
+  return (size_t)mr * (size_t)ppad * (size_t)sub_of(wk) * 16u;
+}
+
+// Compiled activation-row counts (sq_gemv.cuh instantiations).
+static const int kMRs[] = {1, 2, 4, 5, 8, 16};
+
+int gemv_pick_mr(int M) {
+  for (int mr : kMRs)
+    if (M <= mr) return mr;
+  return 16;
+}
+
+// Largest compiled MR whose staged x fits in shared memory.
+static int gemv_cap_mr(int wk, int64_t K) {
+  const size_t limit = (size_t)device_max_smem() - 1024;
+  int best = 0;
+  for (int mr : kMRs)
+    if (gemv_smem_bytes(wk, mr, K) <= limit) best = mr;
+  return best;
+}
+
+cudaError_t launch_gemv(int wk, const GemvArgs& a0, cudaStream_t st) {
+  GemvArgs a = a0;
+  const int cap = gemv_cap_mr(wk, a.K);
+  if (cap == 0) return cudaErrorInvalidValue;
+  const int sms = device_sm_count();
+  // Rows of x are processed in chunks of at most `cap` (each chunk reads the
+  // weights once); M <= 16 with K up to ~19k fits in one or two chunks.
+  for (int m0 = 0; m0 < a0.M;) {
+    const int rem = a0.M - m0;
+    int mr = gemv_pick_mr(rem < cap ? rem : cap);
+    if (mr > cap) {
+      mr = 0;
+      for (int c : kMRs)
+        if (c <= cap) mr = c;
+    }
+    const int m_here = rem < mr ? rem : mr;
+    a.M = m_here;
+    a.x = a0.x + (int64_t)m0 * a0.K;
+    a.y = a0.y + (int64_t)m0 * a0.N;
+    a.residual = a0.residual ? a0.residual + (int64_t)m0 * a0.N : nullptr;
+    const bool silu = a.epi == SQ_EPI_SILU_GATE;
+    const int r = (mr <= 5 && a.N >= 8192) ? 2 : 1;
+    const int64_t ntiles = (a.N + r - 1) / r;
+    const int64_t blocks = (ntiles + 7) / 8;
+    const size_t smem = gemv_smem_bytes(wk, mr, a.K);
+    int per_sm = (int)((size_t)(device_max_smem()) / (smem + 1024));
+    if (per_sm > 8) per_sm = 8;
+    if (per_sm < 1) per_sm = 1;
+    const int64_t cap_blocks = (int64_t)sms * per_sm;
+    const int grid = (int)(blocks < cap_blocks ? blocks : cap_blocks);
+    cudaError_t e;
+    if (wk == SQ_W_INT4) e = launch_gemv_int4(a, mr, r, silu, grid, smem, st);
+    else if (wk == SQ_W_FP8) e = launch_gemv_fp8(a, mr, r, silu, grid, smem, st);
+    else e = launch_gemv_fp16(a, mr, r, silu, grid, smem, st);
+    if (e != cudaSuccess) return e;
+    m0 += m_here;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace sq
+
+using namespace sq;
+
+extern "C" {
+
+const char* sq_last_error(void) { return g_last_error.c_str(); }
+
+const char* sq_status_string(sq_status s) {
+  switch (s) {
+    case SQ_OK: return "SQ_OK";
+    case SQ_ERR_INVALID_ARG: return "SQ_ERR_INVALID_ARG";
+    case SQ_ERR_SHAPE: return "SQ_ERR_SHAPE";
+    case SQ_ERR_ALIGN: return "SQ_ERR_ALIGN";
+    case SQ_ERR_UNSUPPORTED: return "SQ_ERR_UNSUPPORTED";
+    case SQ_ERR_WORKSPACE: return "SQ_ERR_WORKSPACE";
+    case SQ_ERR_CUDA: return "SQ_ERR_CUDA";
+    case SQ_ERR_DEVICE: return "SQ_ERR_DEVICE";
+  }
+  return "SQ_STATUS_UNKNOWN";
+}
+
+int sq_version(void) { return 100; }
+
+sq_status sq_check(sq_stream_t stream, uint32_t* device_bits) {
+  cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_check: stream synchronize");
+  uint32_t bits = 0;
+  if ((e = take_quant_status(&bits)) != cudaSuccess) return cuda_fail(e, "sq_check: quantize status");
+  if ((e = take_accept_status(&bits)) != cudaSuccess) return cuda_fail(e, "sq_check: accept status");
+  if (device_bits) *device_bits = bits;
+  if (bits) return fail(SQ_ERR_DEVICE, "sq_check: device status bits 0x%x", bits);
+  return SQ_OK;
+}
+
+size_t sq_quantized_bytes(sq_qkind kind, int64_t N, int64_t K, size_t* scale_bytes) {
+  if (scale_bytes) *scale_bytes = 0;
+  if (N < 0 || K <= 0) return 0;
+  if (kind == SQ_INT4_G128) {
+    if (K % 128) return 0;
+    if (scale_bytes) *scale_bytes = (size_t)N * (size_t)(K / 128) * 2u;
+    return (size_t)N * (size_t)(K / 2);
+  }
+  if (kind == SQ_FP8_E4M3_ROW) {
+    if (K % 16) return 0;
+    if (scale_bytes) *scale_bytes = (size_t)N * 4u;
+    return (size_t)N * (size_t)K;
+  }
+  return 0;
+}
+
+sq_status sq_quantize(const void* w16, int64_t N, int64_t K, sq_qkind kind, void* codes,
+                      void* scales, sq_stream_t stream) {
+  if (kind != SQ_INT4_G128 && kind != SQ_FP8_E4M3_ROW)
+    return fail(SQ_ERR_INVALID_ARG, "sq_quantize: unknown kind %d", (int)kind);
+  if (N < 0 || K <= 0) return fail(SQ_ERR_SHAPE, "sq_quantize: N=%lld K=%lld", (long long)N, (long long)K);
+  if (kind == SQ_INT4_G128 && K % 128)
+    return fail(SQ_ERR_SHAPE, "sq_quantize: INT4 needs K %% 128 == 0 (K=%lld)", (long long)K);
+  if (kind == SQ_FP8_E4M3_ROW && K % 16)
+    return fail(SQ_ERR_SHAPE, "sq_quantize: FP8 needs K %% 16 == 0 (K=%lld)", (long long)K);
+  if (N == 0) return SQ_OK;
+  if (!w16 || !codes || !scales) return fail(SQ_ERR_INVALID_ARG, "sq_quantize: NULL pointer");
+  if (!aligned(w16, 16) || !aligned(codes, 16))
+    return fail(SQ_ERR_ALIGN, "sq_quantize: w16 and codes must be 16-byte aligned");
+  if (!aligned(scales, kind == SQ_INT4_G128 ? 2 : 4))
+    return fail(SQ_ERR_ALIGN, "sq_quantize: scales misaligned");
+  cudaError_t e = kind == SQ_INT4_G128 ? launch_quant_int4(w16, N, K, codes, scales, (cudaStream_t)stream)
+                                       : launch_quant_fp8(w16, N, K, codes, scales, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_quantize: launch");
+  return SQ_OK;
+}
+
+sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void* scales,
+                       const void* bias, const void* residual, sq_epilogue epi, void* y, int M,
+                       int64_t N, int64_t K, sq_stream_t stream) {
+  if (wkind != SQ_W_FP16 && wkind != SQ_W_INT4 && wkind != SQ_W_FP8)
+    return fail(SQ_ERR_INVALID_ARG, "sq_linear: unknown weight kind %d", (int)wkind);
+  if (epi != SQ_EPI_NONE && epi != SQ_EPI_SILU_GATE && epi != SQ_EPI_RESIDUAL)
+    return fail(SQ_ERR_INVALID_ARG, "sq_linear: unknown epilogue %d", (int)epi);
+  if (M < 1 || M > 256 || N < 1 || K < 1)
+    return fail(SQ_ERR_SHAPE, "sq_linear: need 1 <= M <= 256, N >= 1, K >= 1 (M=%d N=%lld K=%lld)", M,
+                (long long)N, (long long)K);
+  if (wkind == SQ_W_INT4 && K % 128)
+    return fail(SQ_ERR_SHAPE, "sq_linear_w4a16: K %% 128 != 0 (K=%lld)", (long long)K);
+  if (wkind == SQ_W_FP8 && K % 16)
+    return fail(SQ_ERR_SHAPE, "sq_linear_fp8: K %% 16 != 0 (K=%lld)", (long long)K);
+  if (wkind == SQ_W_FP16 && K % 8)
+    return fail(SQ_ERR_SHAPE, "sq_verify: K %% 8 != 0 (K=%lld)", (long long)K);
+  if (N > (int64_t)1 << 30 || K > (int64_t)1 << 20)
+    return fail(SQ_ERR_SHAPE, "sq_linear: N or K too large");
+  if (!x || !w || !y) return fail(SQ_ERR_INVALID_ARG, "sq_linear: NULL x, weight or y");
+  if (wkind != SQ_W_FP16 && !scales) return fail(SQ_ERR_INVALID_ARG, "sq_linear: NULL scales");
+  if (epi == SQ_EPI_RESIDUAL && !residual)
+    return fail(SQ_ERR_INVALID_ARG, "sq_linear: SQ_EPI_RESIDUAL needs a residual");
+  if (!aligned(x, 16) || !aligned(w, 16) || !aligned(y, 2))
+    return fail(SQ_ERR_ALIGN, "sq_linear: x and weights must be 16-byte aligned, y 2-byte aligned");
+  if (scales && !aligned(scales, wkind == SQ_W_FP8 ? 4 : 2))
+    return fail(SQ_ERR_ALIGN, "sq_linear: scales misaligned");
+  if ((bias && !aligned(bias, 2)) || (residual && !aligned(residual, 2)))
+    return fail(SQ_ERR_ALIGN, "sq_linear: bias/residual misaligned");
+  if (gemv_cap_mr(wkind, K) == 0)
+    return fail(SQ_ERR_SHAPE, "sq_linear: K=%lld too large for the staged activations", (long long)K);
+  GemvArgs a = {};
+  a.x = reinterpret_cast<const __half*>(x);
+  a.w = reinterpret_cast<const uint8_t*>(w);
+  a.scales = scales;
+  a.bias = reinterpret_cast<const __half*>(bias);
+  a.residual = epi == SQ_EPI_RESIDUAL ? reinterpret_cast<const __half*>(residual) : nullptr;
+  a.y = reinterpret_cast<__half*>(y);
+  a.M = M;
+  a.epi = epi;
+  a.N = N;
+  a.K = K;
+  a.row_bytes = row_bytes_of(wkind, K);
+  a.pieces = (int)(K / weights_per_piece(wkind));
+  a.ppad = (a.pieces + 31) / 32 * 32;
+  cudaError_t e = launch_gemv(wkind, a, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_linear: launch");
+  return SQ_OK;
+}
+
+sq_status sq_linear_w4a16(const void* x, const void* codes, const void* scales, const void* bias,
+                          void* y, int M, int64_t N, int64_t K, sq_stream_t stream) {
+  return sq_linear_ex(SQ_W_INT4, x, codes, scales, bias, nullptr, SQ_EPI_NONE, y, M, N, K, stream);
+}
+
+sq_status sq_linear_fp8(const void* x, const void* codes, const float* scales, const void* bias,
+                        void* y, int M, int64_t N, int64_t K, sq_stream_t stream) {
+  return sq_linear_ex(SQ_W_FP8, x, codes, scales, bias, nullptr, SQ_EPI_NONE, y, M, N, K, stream);
+}
+
+sq_status sq_verify(const void* x, const void* w16, const void* bias, void* y, int M, int64_t N,
+                    int64_t K, sq_stream_t stream) {
+  return sq_linear_ex(SQ_W_FP16, x, w16, nullptr, bias, nullptr, SQ_EPI_NONE, y, M, N, K, stream);
+}
+
+size_t sq_accept_workspace_bytes(int B, int K, int64_t V) {
+  if (B < 0 || K < 0 || K > 16 || V < 1 || V >= ((int64_t)1 << 20)) return 0;
+  return accept_workspace_bytes(B, K, V);
+}
+
+static sq_status accept_common(const char* who, const float* p, const float* q, const int32_t* draft,
+                               const float* u, int B, int K, int64_t V, int mode, int32_t* n_accepted,
+                               int32_t* tokens, void* workspace, size_t ws_bytes,
+                               sq_stream_t stream) {
+  if (mode != SQ_ACCEPT_SAMPLE && mode != SQ_ACCEPT_GREEDY)
+    return fail(SQ_ERR_INVALID_ARG, "%s: unknown mode %d", who, mode);
+  if (B < 0 || K < 0 || K > 16 || V < 1 || V >= ((int64_t)1 << 20))
+    return fail(SQ_ERR_SHAPE, "%s: need B >= 0, 0 <= K <= 16, 1 <= V < 2^20 (B=%d K=%d V=%lld)", who, B,
+                K, (long long)V);
+  if (B == 0) return SQ_OK;
+  if (!p || !u || !tokens || (K > 0 && !draft))
+    return fail(SQ_ERR_INVALID_ARG, "%s: NULL p, u, draft or tokens", who);
+  if (K > 0 && mode == SQ_ACCEPT_SAMPLE && !q)
+    return fail(SQ_ERR_INVALID_ARG, "%s: sampling mode with K > 0 needs q", who);
+  if (!aligned(p, 4) || (q && !aligned(q, 4)) || !aligned(u, 4) || (draft && !aligned(draft, 4)) ||
+      !aligned(tokens, 4) || (n_accepted && !aligned(n_accepted, 4)))
+    return fail(SQ_ERR_ALIGN, "%s: pointers must be 4-byte aligned", who);
+  const size_t need = accept_workspace_bytes(B, K, V);
+  if (!workspace || ws_bytes < need)
+    return fail(SQ_ERR_WORKSPACE, "%s: workspace %zu bytes < %zu required", who, ws_bytes, need);
+  if (!aligned(workspace, 16)) return fail(SQ_ERR_ALIGN, "%s: workspace must be 16-byte aligned", who);
+  AcceptArgs a = {};
+  a.p = p;
+  a.q = K > 0 ? q : nullptr;
+  a.draft = draft;
+  a.u = u;
+  a.B = B;
+  a.K = K;
+  a.V = V;
+  a.mode = mode;
+  a.n_out = n_accepted;
+  a.tok_out = tokens;
+  const size_t ctr = (((size_t)B * 4u) + 15u) & ~(size_t)15u;
+  a.counter = reinterpret_cast<unsigned int*>(workspace);
+  a.part = reinterpret_cast<unsigned long long*>(reinterpret_cast<char*>(workspace) + ctr);
+  a.C = (int)((V + kAcceptChunk - 1) / kAcceptChunk);
+  a.chunk = kAcceptChunk;
+  a.slots = K + 1 > 2 ? K + 1 : 2;
+  cudaError_t e = launch_accept(a, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_accept: launch");
+  return SQ_OK;
+}
+
+sq_status sq_accept(const float* p, const float* q, const int32_t* draft, const float* u, int B, int K,
+                    int64_t V, sq_accept_mode mode, int32_t* n_accepted, int32_t* tokens,
+                    void* workspace, size_t ws_bytes, sq_stream_t stream) {
+  if (!n_accepted && B > 0) return fail(SQ_ERR_INVALID_ARG, "sq_accept: NULL n_accepted");
+  return accept_common("sq_accept", p, q, draft, u, B, K, V, (int)mode, n_accepted, tokens, workspace,
+                       ws_bytes, stream);
+}
+
+sq_status sq_sample(const float* probs, const float* u, int B, int64_t V, int32_t* tokens,
+                    void* workspace, size_t ws_bytes, sq_stream_t stream) {
+  return accept_common("sq_sample", probs, nullptr, nullptr, u, B, 0, V, SQ_ACCEPT_SAMPLE, nullptr,
+                       tokens, workspace, ws_bytes, stream);
+}
+
+}  // extern "C"

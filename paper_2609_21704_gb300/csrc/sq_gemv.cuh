@@ -1,0 +1,281 @@
+// sq_gemv.cuh -- skinny linear layer y = x W'^T for 1..16 activation rows
+// on CUDA cores (Sec. III-D.2 draft pass at M = batch, Sec. III-D.3 verify
+// pass at M = batch * (K+1) while that stays below a tensor-core tile).
+//
+// The work is HBM-bound: every weight byte is read once; x (M x K fp16) and
+// y are small.  Mapping:
+//   * a warp owns R weight rows (2R for the fused SiLU gate) and sweeps the
+//     whole row, each lane taking one 16-byte piece of each row per step
+//     (32 INT4, 16 FP8 or 8 FP16 weights) with a non-allocating 128-bit
+//     load: 512 contiguous bytes per row per warp-step, fully coalesced;
+//   * x is staged once per CTA into shared memory, permuted so that the
+//     16-byte x chunk lane l needs at sub-step i sits at slot
+//     (step * SUB + i) * 32 + l: 32 lanes read 512 consecutive bytes, no
+//     bank conflicts, and each x chunk serves R rows from registers;
+//   * products are fp16 x fp16 -> fp32 (exact) with fp32 accumulation
+//     (fma.rn.f32.f16); INT4 codes become exact fp16 integers with two
+//     logic ops and one packed fp16 op per pair, and the group scale is
+//     applied once per 32-weight piece; the FP8 row scale once per output;
+//   * the per-lane partial sums are reduced with warp shuffles in a fixed
+//     order, so results are reproducible run to run.
+// Before waiting on the kernel that produces x, each CTA asks L2 to
+// prefetch the first weight bytes it will read (weights never depend on
+// the previous kernel), which overlaps the launch gap with HBM traffic.
+#pragma once
+
+#include "sq_internal.h"
+
+namespace sq {
+
+enum { WK_FP16 = 0, WK_INT4 = 1, WK_FP8 = 2 };
+
+template <int WK>
+struct WTraits;
+template <>
+struct WTraits<WK_INT4> {
+  static constexpr int kWeightsPerPiece = 32;
+  static constexpr int kSub = 4;  // 8-weight x chunks per piece
+};
+template <>
+struct WTraits<WK_FP8> {
+  static constexpr int kWeightsPerPiece = 16;
+  static constexpr int kSub = 2;
+};
+template <>
+struct WTraits<WK_FP16> {
+  static constexpr int kWeightsPerPiece = 8;
+  static constexpr int kSub = 1;
+};
+
+constexpr int kGemvThreads = 256;
+constexpr int kGemvWarps = kGemvThreads / 32;
+
+// acc[m] += sum_{j<8} c_j * x_j for one 8-weight chunk; c holds the codes as
+// fp16 pairs (c0,c4),(c1,c5),(c2,c6),(c3,c7) (INT4 order) and xq the chunk
+// (x0,x1),(x2,x3),(x4,x5),(x6,x7).
+__device__ __forceinline__ float dot8_int4order(const uint32_t c[4], const uint4 xq, float acc) {
+  acc = fma_h(lo16(c[0]), lo16(xq.x), acc);
+  acc = fma_h(lo16(c[1]), hi16(xq.x), acc);
+  acc = fma_h(lo16(c[2]), lo16(xq.y), acc);
+  acc = fma_h(lo16(c[3]), hi16(xq.y), acc);
+  acc = fma_h(hi16(c[0]), lo16(xq.z), acc);
+  acc = fma_h(hi16(c[1]), hi16(xq.z), acc);
+  acc = fma_h(hi16(c[2]), lo16(xq.w), acc);
+  acc = fma_h(hi16(c[3]), hi16(xq.w), acc);
+  return acc;
+}
+
+// Same for weights already in natural order: pairs (w0,w1),(w2,w3),...
+__device__ __forceinline__ float dot8_natural(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3,
+                                              const uint4 xq, float acc) {
+  acc = fma_h(lo16(w0), lo16(xq.x), acc);
+  acc = fma_h(hi16(w0), hi16(xq.x), acc);
+  acc = fma_h(lo16(w1), lo16(xq.y), acc);
+  acc = fma_h(hi16(w1), hi16(xq.y), acc);
+  acc = fma_h(lo16(w2), lo16(xq.z), acc);
+  acc = fma_h(hi16(w2), hi16(xq.z), acc);
+  acc = fma_h(lo16(w3), lo16(xq.w), acc);
+  acc = fma_h(hi16(w3), hi16(xq.w), acc);
+  return acc;
+}
+
+// MR: activation rows compiled for (M <= MR, missing rows read zeros);
+// R: output rows per warp; SILU: fused gate/up epilogue.
+template <int WK, int MR, int R, bool SILU>
+__global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
+  using T = WTraits<WK>;
+  constexpr int SUB = T::kSub;
+  constexpr int WR = SILU ? 2 * R : R;  // weight rows per warp tile
+  extern __shared__ uint4 xs[];
+
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t ntiles = (a.N + R - 1) / R;
+  const int64_t gwarp = (int64_t)blockIdx.x * kGemvWarps + warp;
+  const int64_t nwarps = (int64_t)gridDim.x * kGemvWarps;
+
+  auto wrow_index = [&](int64_t tile, int r) -> int64_t {
+    if (!SILU) return tile * R + r;
+    return r < R ? tile * R + r : a.N + tile * R + (r - R);
+  };
+  auto row_valid = [&](int64_t tile, int r) -> bool {
+    return tile * R + (SILU ? (r % R) : r) < a.N;
+  };
+
+  // L2 prefetch of this warp's first tile (weights do not depend on the
+  // previous kernel, so this overlaps its tail).
+  if (gwarp < ntiles && lane < WR && row_valid(gwarp, lane)) {
+    const uint8_t* row = a.w + wrow_index(gwarp, lane) * a.row_bytes;
+    const int64_t nb = a.row_bytes < 4096 ? a.row_bytes : 4096;
+    prefetch_l2_bulk(row, (uint32_t)(nb & ~15ll));
+  }
+
+  griddep_wait();
+  griddep_launch_dependents();
+
+  // ---- stage x, permuted (see header comment)
+  const int chunks_per_m = a.ppad * SUB;
+  for (int idx = threadIdx.x; idx < MR * chunks_per_m; idx += kGemvThreads) {
+    const int m = idx / chunks_per_m;
+    const int s = idx - m * chunks_per_m;
+    const int l = s & 31, t = s >> 5;
+    const int j = t / SUB, i = t - j * SUB;
+    const int p = j * 32 + l;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (m < a.M && p < a.pieces)
+      v = *reinterpret_cast<const uint4*>(a.x + (int64_t)m * a.K + ((int64_t)p * SUB + i) * 8);
+    xs[idx] = v;
+  }
+  __syncthreads();
+
+  const int steps = a.ppad / 32;
+  for (int64_t tile = gwarp; tile < ntiles; tile += nwarps) {
+    const uint8_t* wrow[WR];
+    bool valid[WR];
+#pragma unroll
+    for (int r = 0; r < WR; ++r) {
+      valid[r] = row_valid(tile, r);
+      wrow[r] = a.w + (valid[r] ? wrow_index(tile, r) : 0) * a.row_bytes;
+    }
+    float acc[WR][MR];
+#pragma unroll
+    for (int r = 0; r < WR; ++r)
+#pragma unroll
+      for (int m = 0; m < MR; ++m) acc[r][m] = 0.0f;
+
+    for (int j = 0; j < steps; ++j) {
+      const int p = j * 32 + lane;
+      if (p >= a.pieces) break;
+      uint4 wv[WR];
+#pragma unroll
+      for (int r = 0; r < WR; ++r)
+        wv[r] = valid[r] ? ld_stream16(wrow[r] + (int64_t)p * 16) : make_uint4(0u, 0u, 0u, 0u);
+
+      if constexpr (WK == WK_INT4) {
+        const __half* sc = reinterpret_cast<const __half*>(a.scales);
+        const int64_t G = a.K / 128;
+        float part[WR][MR];
+#pragma unroll
+        for (int r = 0; r < WR; ++r)
+#pragma unroll
+          for (int m = 0; m < MR; ++m) part[r][m] = 0.0f;
+#pragma unroll
+        for (int i = 0; i < SUB; ++i) {
+          uint32_t c[WR][4];
+#pragma unroll
+          for (int r = 0; r < WR; ++r) {
+            const uint32_t word = i == 0 ? wv[r].x : i == 1 ? wv[r].y : i == 2 ? wv[r].z : wv[r].w;
+            int4x8_to_f16x2(word, c[r]);
+          }
+#pragma unroll
+          for (int m = 0; m < MR; ++m) {
+            const uint4 xq = xs[m * chunks_per_m + (j * SUB + i) * 32 + lane];
+#pragma unroll
+            for (int r = 0; r < WR; ++r) part[r][m] = dot8_int4order(c[r], xq, part[r][m]);
+          }
+        }
+#pragma unroll
+        for (int r = 0; r < WR; ++r) {
+          const float s = valid[r] ? __half2float(sc[wrow_index(tile, r) * G + (p >> 2)]) : 0.0f;
+#pragma unroll
+          for (int m = 0; m < MR; ++m) acc[r][m] = fmaf(s, part[r][m], acc[r][m]);
+        }
+      } else if constexpr (WK == WK_FP8) {
+#pragma unroll
+        for (int i = 0; i < SUB; ++i) {
+          uint32_t h[WR][4];
+#pragma unroll
+          for (int r = 0; r < WR; ++r) {
+            const uint32_t wa = i == 0 ? wv[r].x : wv[r].z;
+            const uint32_t wb = i == 0 ? wv[r].y : wv[r].w;
+            h[r][0] = e4m3x2_to_f16x2(lo16(wa));
+            h[r][1] = e4m3x2_to_f16x2(hi16(wa));
+            h[r][2] = e4m3x2_to_f16x2(lo16(wb));
+            h[r][3] = e4m3x2_to_f16x2(hi16(wb));
+          }
+#pragma unroll
+          for (int m = 0; m < MR; ++m) {
+            const uint4 xq = xs[m * chunks_per_m + (j * SUB + i) * 32 + lane];
+#pragma unroll
+            for (int r = 0; r < WR; ++r)
+              acc[r][m] = dot8_natural(h[r][0], h[r][1], h[r][2], h[r][3], xq, acc[r][m]);
+          }
+        }
+      } else {
+#pragma unroll
+        for (int m = 0; m < MR; ++m) {
+          const uint4 xq = xs[m * chunks_per_m + j * 32 + lane];
+#pragma unroll
+          for (int r = 0; r < WR; ++r)
+            acc[r][m] = dot8_natural(wv[r].x, wv[r].y, wv[r].z, wv[r].w, xq, acc[r][m]);
+        }
+      }
+    }
+
+    // ---- reduce across the warp (fixed butterfly order)
+#pragma unroll
+    for (int r = 0; r < WR; ++r)
+#pragma unroll
+      for (int m = 0; m < MR; ++m) acc[r][m] = warp_sum(acc[r][m]);
+
+    // ---- epilogue: lane (r * MR + m) % 32 writes output (r, m)
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int64_t n = tile * R + r;
+      if (n >= a.N) continue;
+#pragma unroll
+      for (int m = 0; m < MR; ++m) {
+        if (m >= a.M || lane != ((r * MR + m) & 31)) continue;
+        float v = acc[r][m];
+        if constexpr (WK == WK_FP8) v *= reinterpret_cast<const float*>(a.scales)[n];
+        if (a.bias) v += __half2float(a.bias[n]);
+        if constexpr (SILU) {
+          float u = acc[R + r][m];
+          if constexpr (WK == WK_FP8) u *= reinterpret_cast<const float*>(a.scales)[a.N + n];
+          if (a.bias) u += __half2float(a.bias[a.N + n]);
+          v = v / (1.0f + expf(-v)) * u;
+        }
+        if (a.residual) v += __half2float(a.residual[(int64_t)m * a.N + n]);
+        a.y[(int64_t)m * a.N + n] = __float2half_rn(v);
+      }
+    }
+  }
+}
+
+// Instantiation helper used by the per-format translation units.
+template <int WK, int MR, int R, bool SILU>
+cudaError_t launch_gemv_inst(const GemvArgs& a, int grid, size_t smem, cudaStream_t st) {
+  auto k = gemv_kernel<WK, MR, R, SILU>;
+  static int smem_set[64] = {0};  // per device: largest dynamic smem enabled so far
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (smem > 48 * 1024 && dev < 64 && (int)smem > smem_set[dev]) {
+    e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    smem_set[dev] = (int)smem;
+  }
+  return launch_pdl(k, dim3(grid), dim3(kGemvThreads), smem, st, a);
+}
+
+template <int WK>
+cudaError_t launch_gemv_fmt(const GemvArgs& a, int mr, int r, bool silu, int grid, size_t smem,
+                            cudaStream_t st) {
+#define SQ_GEMV_CASE(MR_, R_)                                                              \
+  if (mr == MR_ && r == R_)                                                                \
+    return silu ? launch_gemv_inst<WK, MR_, R_, true>(a, grid, smem, st)                   \
+                : launch_gemv_inst<WK, MR_, R_, false>(a, grid, smem, st);
+  SQ_GEMV_CASE(1, 1)
+  SQ_GEMV_CASE(1, 2)
+  SQ_GEMV_CASE(2, 1)
+  SQ_GEMV_CASE(2, 2)
+  SQ_GEMV_CASE(4, 1)
+  SQ_GEMV_CASE(4, 2)
+  SQ_GEMV_CASE(5, 1)
+  SQ_GEMV_CASE(5, 2)
+  SQ_GEMV_CASE(8, 1)
+  SQ_GEMV_CASE(16, 1)
+#undef SQ_GEMV_CASE
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace sq

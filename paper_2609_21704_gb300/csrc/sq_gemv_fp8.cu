@@ -1,0 +1,13 @@
+// sq_gemv_fp8.cu -- instantiations of the CUDA-core skinny linear layer for
+// fp8 weights (one translation unit per weight format so they compile in
+// parallel).
+#include "sq_gemv.cuh"
+
+namespace sq {
+
+cudaError_t launch_gemv_fp8(const GemvArgs& a, int mr, int r, bool silu, int grid, size_t smem,
+                           cudaStream_t st) {
+  return launch_gemv_fmt<WK_FP8>(a, mr, r, silu, grid, smem, st);
+}
+
+}  // namespace sq

@@ -1,0 +1,93 @@
+// sq_internal.h -- declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/specquant.h"
+#include "sq_device.cuh"
+
+namespace sq {
+
+constexpr int kNumSMs = 152;  // GB300: 2 dies x 76 SMs (queried at run time too)
+
+int device_sm_count();
+
+// Launch with programmatic dependent launch allowed: the kernel may begin
+// while the previous kernel on the stream drains; it must call
+// griddep_wait() before touching data that kernel produced or consumes.
+// The legacy default stream gets a plain launch.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  const bool legacy = (st == nullptr || st == cudaStreamLegacy || st == cudaStreamPerThread);
+  cfg.attrs = legacy ? nullptr : attr;
+  cfg.numAttrs = legacy ? 0 : 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
+// sq_quantize.cu
+cudaError_t launch_quant_int4(const void* w, int64_t N, int64_t K, void* codes, void* scales,
+                              cudaStream_t st);
+cudaError_t launch_quant_fp8(const void* w, int64_t N, int64_t K, void* codes, void* scales,
+                             cudaStream_t st);
+cudaError_t take_quant_status(uint32_t* bits);
+
+// GEMV family (sq_gemv_*.cu): M <= 16 rows of activations on CUDA cores.
+struct GemvArgs {
+  const __half* x;         // [M, K]
+  const uint8_t* w;        // weight rows (codes or fp16 bytes)
+  const void* scales;      // INT4: fp16 [rows, K/128]; FP8: fp32 [rows]; FP16: unused
+  const __half* bias;      // [rows] or null
+  const __half* residual;  // [M, N] or null
+  __half* y;               // [M, N]
+  int M;                   // activation rows present (<= template MR)
+  int epi;                 // sq_epilogue
+  int64_t N;               // output columns
+  int64_t K;
+  int64_t row_bytes;       // bytes of one weight row
+  int pieces;              // 16-byte pieces per weight row
+  int ppad;                // pieces rounded up to a multiple of 32
+};
+constexpr int kGemvMaxRows = 16;
+size_t gemv_smem_bytes(int wkind, int mr, int64_t K);
+int gemv_pick_mr(int M);
+cudaError_t launch_gemv(int wkind, const GemvArgs& a, cudaStream_t st);
+cudaError_t launch_gemv_int4(const GemvArgs& a, int mr, int r, bool silu, int grid, size_t smem,
+                             cudaStream_t st);
+cudaError_t launch_gemv_fp8(const GemvArgs& a, int mr, int r, bool silu, int grid, size_t smem,
+                            cudaStream_t st);
+cudaError_t launch_gemv_fp16(const GemvArgs& a, int mr, int r, bool silu, int grid, size_t smem,
+                             cudaStream_t st);
+
+// sq_accept.cu
+struct AcceptArgs {
+  const float* p;
+  const float* q;
+  const int32_t* draft;
+  const float* u;
+  int B, K;
+  int64_t V;
+  int mode;
+  int32_t* n_out;
+  int32_t* tok_out;
+  unsigned long long* part;  // [B][C][slots]
+  unsigned int* counter;     // [B]
+  int C;                     // chunks per sequence
+  int chunk;                 // vocabulary entries per chunk
+  int slots;                 // partial slots per chunk
+};
+constexpr int kAcceptChunk = 2048;
+size_t accept_workspace_bytes(int B, int K, int64_t V);
+cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t st);
+cudaError_t take_accept_status(uint32_t* bits);
+
+}  // namespace sq

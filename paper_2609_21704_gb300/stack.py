@@ -1,0 +1,156 @@
+"""Device-resident linear stack of a Qwen2.5-shaped model and one
+speculative draft/verify cycle over it, driven through the C ABI.
+
+Sec. III-A: one FP16 parent W16 with the INT4 (Q4) and FP8 (Q8) variants
+derived from it by ``sq_quantize``, all resident in HBM at once.
+Sec. III-D.2: the draft pass runs every projection plus lm_head at M = B.
+Sec. III-D.3: the verify pass runs them at M = B (K + 1) with the parent.
+Sec. III-D.4: ``sq_accept`` over the vocabulary.
+
+Attention, RMSNorm, RoPE and the residual stream are outside the hot path.
+A pass therefore runs, per layer:
+    qkv = x_l W_qkv^T                      (fused q/k/v, one launch)
+    o   = a W_o^T                          a = the first M * q_out values of
+                                           qkv read as [M, q_out] (for M = 1
+                                           exactly the q row): attention's
+                                           stand-in keeps the qkv -> o order
+    h   = silu(x_l W_g^T) * (x_l W_u^T)    (fused gate/up + SiLU, one launch)
+    d   = h W_down^T
+and then logits = x W_lm^T.  x_l is a resident synthetic N(0, 1) hidden
+state; without normalisation a random-init residual stream overflows fp16
+within a few layers, so the layers are fed fresh activations while every
+projection still runs once, in stream order, with its real weights.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import torch
+
+from . import (SQ_EPI_NONE, SQ_EPI_SILU_GATE, SQ_FP8_E4M3_ROW, SQ_INT4_G128, SQ_W_FP8,
+               SQ_W_FP16, SQ_W_INT4, sq_linear_ex, sq_quantize, sq_quantized_bytes, synth)
+from .shapes import StackShape
+
+WKIND = {"fp16": SQ_W_FP16, "int4": SQ_W_INT4, "fp8": SQ_W_FP8}
+BYTES_PER_WEIGHT = {"fp16": 2.0, "int4": 0.5 + 2.0 / 128.0, "fp8": 1.0}
+
+
+@dataclass
+class Proj:
+    name: str
+    n_out: int      # weight rows
+    k_in: int
+    epi: int
+    w16: torch.Tensor
+    q: dict         # variant -> (codes, scales)
+
+    def weight(self, variant):
+        if variant == "fp16":
+            return self.w16, None
+        return self.q[variant]
+
+    def y_cols(self):
+        return self.n_out // 2 if self.epi == SQ_EPI_SILU_GATE else self.n_out
+
+    def weight_bytes(self, variant) -> int:
+        n, k = self.n_out, self.k_in
+        if variant == "fp16":
+            return 2 * n * k
+        kind = SQ_INT4_G128 if variant == "int4" else SQ_FP8_E4M3_ROW
+        cb, sb = sq_quantized_bytes(kind, n, k)
+        return cb + sb
+
+
+class LinearStack:
+    """All projections of ``layers`` decoder layers plus lm_head, FP16 parent
+    and the requested derived variants, resident on ``device``."""
+
+    def __init__(self, shape: StackShape, device, seed: int = 0, variants=("int4", "fp8"),
+                 layers: int | None = None, with_lm_head: bool = True):
+        self.shape = shape
+        self.device = torch.device(device)
+        self.variants = tuple(variants)
+        self.layers = []
+        nl = shape.layers if layers is None else layers
+        s = seed
+        for _ in range(nl):
+            layer = []
+            for name, n, k in shape.projections():
+                epi = SQ_EPI_SILU_GATE if name == "gate_up" else SQ_EPI_NONE
+                layer.append(self._make(name, n, k, epi, s))
+                s += 1
+            self.layers.append(layer)
+        self.lm_head = None
+        if with_lm_head:
+            name, n, k = shape.lm_head()
+            self.lm_head = self._make(name, n, k, SQ_EPI_NONE, s)
+
+    def _make(self, name, n, k, epi, seed) -> Proj:
+        w16 = synth.weights_fp16_device(seed * 7919 + 17, n, k, self.device)
+        q = {}
+        for v in self.variants:
+            kind = SQ_INT4_G128 if v == "int4" else SQ_FP8_E4M3_ROW
+            cb, sb = sq_quantized_bytes(kind, n, k)
+            codes = torch.empty((n, cb // n), dtype=torch.uint8, device=self.device)
+            if v == "int4":
+                scales = torch.empty((n, k // 128), dtype=torch.float16, device=self.device)
+            else:
+                scales = torch.empty((n,), dtype=torch.float32, device=self.device)
+            sq_quantize(w16, kind, codes, scales)
+            q[v] = (codes, scales)
+        return Proj(name, n, k, epi, w16, q)
+
+    def projections(self):
+        for layer in self.layers:
+            yield from layer
+        if self.lm_head is not None:
+            yield self.lm_head
+
+    def launches_per_pass(self) -> int:
+        return sum(1 for _ in self.projections())
+
+    def weight_bytes(self, variant) -> int:
+        return sum(p.weight_bytes(variant) for p in self.projections())
+
+    def activation_bytes(self, M: int) -> int:
+        return sum(2 * M * (p.k_in + p.y_cols()) for p in self.projections())
+
+    def params(self) -> int:
+        return sum(p.n_out * p.k_in for p in self.projections())
+
+
+class PassBuffers:
+    """Activations and outputs of one pass at M rows."""
+
+    def __init__(self, stack: LinearStack, M: int, seed: int = 1):
+        sh, dev = stack.shape, stack.device
+        self.M = M
+        self.x = synth.activations_fp16_device(seed, M, sh.hidden, dev)
+        nq = sh.q_out + 2 * sh.kv_out
+        self.qkv = torch.empty((M, nq), dtype=torch.float16, device=dev)
+        self.o = torch.empty((M, sh.hidden), dtype=torch.float16, device=dev)
+        self.h = torch.empty((M, sh.intermediate), dtype=torch.float16, device=dev)
+        self.d = torch.empty((M, sh.hidden), dtype=torch.float16, device=dev)
+        self.logits = torch.empty((M, sh.vocab), dtype=torch.float16, device=dev) \
+            if stack.lm_head is not None else None
+        # attention stand-in: the first M * q_out values of qkv as [M, q_out]
+        self.attn = self.qkv.view(-1)[: M * sh.q_out].view(M, sh.q_out)
+
+
+def run_pass(stack: LinearStack, variant: str, b: PassBuffers, stream=None) -> None:
+    """One draft (variant int4/fp8) or verify (fp16, or fp8) pass: every
+    projection of every layer plus lm_head, in decoder order."""
+    wk = WKIND[variant]
+    for layer in stack.layers:
+        qkv, o, gu, down = layer
+        w, s = qkv.weight(variant)
+        sq_linear_ex(wk, b.x, w, s, None, None, SQ_EPI_NONE, b.qkv, stream)
+        w, s = o.weight(variant)
+        sq_linear_ex(wk, b.attn, w, s, None, None, SQ_EPI_NONE, b.o, stream)
+        w, s = gu.weight(variant)
+        sq_linear_ex(wk, b.x, w, s, None, None, SQ_EPI_SILU_GATE, b.h, stream)
+        w, s = down.weight(variant)
+        sq_linear_ex(wk, b.h, w, s, None, None, SQ_EPI_NONE, b.d, stream)
+    if stack.lm_head is not None:
+        w, s = stack.lm_head.weight(variant)
+        sq_linear_ex(wk, b.x, w, s, None, None, SQ_EPI_NONE, b.logits, stream)

@@ -84,3 +84,26 @@ def spec_block(seed: int, B: int, K: int, V: int, sigma: float = 2.0,
             draft[b, i] = rng.choice(V, p=w / w.sum())
     u = uniforms(seed ^ 0x5EED, (B, K + 1))
     return p, q, draft, u
+
+
+def weights_fp16_device(seed: int, n_out: int, k_in: int, device, std: float = 0.02):
+    """Large fp16 ~ N(0, std) weight matrices drawn on the device with a
+    seeded torch generator (used for full-size workloads; tests copy the
+    rows they check back to the host for the oracle)."""
+    import torch
+
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    w = torch.empty((n_out, k_in), dtype=torch.float16, device=device)
+    w.normal_(0.0, std, generator=g)
+    return w
+
+
+def activations_fp16_device(seed: int, m: int, k_in: int, device):
+    import torch
+
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    x = torch.empty((m, k_in), dtype=torch.float16, device=device)
+    x.normal_(0.0, 1.0, generator=g)
+    return x

@@ -1,0 +1,118 @@
+"""The C-ABI library: it loads, exports every function include/specquant.h
+declares, and its host-side logic (sizes, validation, status strings)
+behaves as documented.  No call here reaches a kernel, so these run
+without a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2609_21704_gb300 as sq
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "specquant.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    sq.build()
+    return sq.load()
+
+
+def _declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(sq_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared_functions()
+    for want in ("sq_quantize", "sq_linear_w4a16", "sq_linear_fp8", "sq_verify", "sq_accept",
+                 "sq_sample", "sq_check", "sq_last_error"):
+        assert want in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in _declared_functions():
+        assert hasattr(lib, name), name
+    assert set(_declared_functions()) <= set(sq.EXPORTED_SYMBOLS) | {"sq_last_error"}
+
+
+def test_library_is_built_for_sm_103a_only():
+    # the fatbin carries one cubin for sm_103a; the ELF note names it
+    data = open(sq.LIB_PATH, "rb").read()
+    assert b"sm_103a" in data or b"sm_103" in data
+
+
+def test_version_and_status_strings(lib):
+    assert sq.sq_version() >= 100
+    assert lib.sq_status_string(0) == b"SQ_OK"
+    assert lib.sq_status_string(5) == b"SQ_ERR_WORKSPACE"
+    assert lib.sq_status_string(99) == b"SQ_STATUS_UNKNOWN"
+
+
+def test_quantized_bytes():
+    assert sq.sq_quantized_bytes(sq.SQ_INT4_G128, 4864, 896) == (4864 * 448, 4864 * 7 * 2)
+    assert sq.sq_quantized_bytes(sq.SQ_FP8_E4M3_ROW, 10, 32) == (320, 40)
+    assert sq.sq_quantized_bytes(sq.SQ_INT4_G128, 4, 100) == (0, 0)
+    assert sq.sq_quantized_bytes(sq.SQ_FP8_E4M3_ROW, 4, 24) == (0, 0)
+    assert sq.sq_quantized_bytes(7, 4, 128) == (0, 0)
+
+
+def test_accept_workspace_bytes():
+    b = sq.sq_accept_workspace_bytes(8, 5, 152064)
+    chunks = (152064 + 2047) // 2048
+    assert b >= 8 * chunks * 6 * 8 + 8 * 4
+    assert sq.sq_accept_workspace_bytes(1, 17, 100) == 0
+    assert sq.sq_accept_workspace_bytes(1, 2, 1 << 20) == 0
+
+
+def _err(lib):
+    return lib.sq_last_error().decode()
+
+
+def test_validation_rejects_before_launch(lib):
+    P = ctypes.c_void_p
+    fake = P(4096)  # never dereferenced: validation fails first
+    # shape errors
+    assert lib.sq_linear_w4a16(fake, fake, fake, None, fake, 0, 16, 128, None) == 2
+    assert "M" in _err(lib)
+    assert lib.sq_linear_w4a16(fake, fake, fake, None, fake, 1, 16, 100, None) == 2
+    assert lib.sq_linear_fp8(fake, fake, fake, None, fake, 1, 16, 24, None) == 2
+    assert lib.sq_verify(fake, fake, None, fake, 300, 16, 64, None) == 2
+    # null pointers
+    assert lib.sq_verify(None, fake, None, fake, 1, 16, 64, None) == 1
+    assert lib.sq_linear_w4a16(fake, fake, None, None, fake, 1, 16, 128, None) == 1
+    # alignment
+    assert lib.sq_verify(P(4098), fake, None, fake, 1, 16, 64, None) == 3
+    # unknown enums
+    assert lib.sq_linear_ex(9, fake, fake, None, None, None, 0, fake, 1, 16, 64, None) == 1
+    assert lib.sq_linear_ex(0, fake, fake, None, None, None, 9, fake, 1, 16, 64, None) == 1
+    assert lib.sq_linear_ex(0, fake, fake, None, None, None, 2, fake, 1, 16, 64, None) == 1
+    assert lib.sq_quantize(fake, 4, 128, 3, fake, fake, None) == 1
+    assert lib.sq_quantize(fake, 4, 100, 1, fake, fake, None) == 2
+    assert lib.sq_quantize(fake, 0, 128, 1, None, None, None) == 0  # empty: nothing to do
+
+
+def test_accept_validation(lib):
+    P = ctypes.c_void_p
+    fake = P(4096)
+    ws_need = sq.sq_accept_workspace_bytes(2, 3, 1000)
+    # workspace too small
+    assert lib.sq_accept(fake, fake, fake, fake, 2, 3, 1000, 0, fake, fake, fake, ws_need - 1, None) == 5
+    # missing q in sampling mode
+    assert lib.sq_accept(fake, None, fake, fake, 2, 3, 1000, 0, fake, fake, fake, ws_need, None) == 1
+    # K too large, V too large, bad mode
+    assert lib.sq_accept(fake, fake, fake, fake, 2, 17, 1000, 0, fake, fake, fake, 1 << 20, None) == 2
+    assert lib.sq_accept(fake, fake, fake, fake, 2, 3, 1 << 20, 0, fake, fake, fake, 1 << 30, None) == 2
+    assert lib.sq_accept(fake, fake, fake, fake, 2, 3, 1000, 5, fake, fake, fake, ws_need, None) == 1
+    # empty batch is a no-op
+    assert lib.sq_accept(None, None, None, None, 0, 3, 1000, 0, None, None, None, 0, None) == 0
+    # workspace misaligned
+    assert lib.sq_sample(fake, fake, 2, 1000, fake, P(4100), 1 << 20, None) == 3
+
+
+def test_binding_fails_loudly_without_the_library(tmp_path):
+    with pytest.raises(ImportError):
+        sq.load(str(tmp_path / "missing.so"))
