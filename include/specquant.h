@@ -26,12 +26,20 @@
  *    draft token outside [0, V), a resampling row without mass) set bits of
  *    a per-device status word that sq_check() reads and clears.
  *  - fp16 means IEEE binary16; E4M3 means the OCP FP8 E4M3 format.
+ *  - Environment: SQ_PDL=0 launches without programmatic dependent launch
+ *    (default: allowed on every stream but the legacy default stream).
  */
 #ifndef SPECQUANT_H
 #define SPECQUANT_H
 
 #include <stddef.h>
 #include <stdint.h>
+
+#if defined(__GNUC__) || defined(__clang__)
+#define SQ_API __attribute__((visibility("default")))
+#else
+#define SQ_API
+#endif
 
 #ifdef __cplusplus
 extern "C" {
@@ -62,16 +70,16 @@ typedef enum { SQ_ACCEPT_SAMPLE = 0, SQ_ACCEPT_GREEDY = 1 } sq_accept_mode;
 #define SQ_DEV_BAD_UNIFORM      0x8u  /* resampling uniform not in [0,1)     */
 
 /* Thread-local text of the last error raised on this host thread. */
-const char* sq_last_error(void);
+SQ_API const char* sq_last_error(void);
 /* Fixed name of a status code. */
-const char* sq_status_string(sq_status s);
+SQ_API const char* sq_status_string(sq_status s);
 /* Library version, major * 10000 + minor * 100 + patch. */
-int sq_version(void);
+SQ_API int sq_version(void);
 
 /* Synchronises `stream`, then reads and clears the device status word of
  * the current device.  Returns SQ_OK, SQ_ERR_DEVICE (bits in *device_bits,
  * which may be NULL) or SQ_ERR_CUDA. */
-sq_status sq_check(sq_stream_t stream, uint32_t* device_bits);
+SQ_API sq_status sq_check(sq_stream_t stream, uint32_t* device_bits);
 
 /* ------------------------------------------------------------------------
  * Sec. III-A.1 / III-A.2: derive the draft variants from the FP16 parent.
@@ -94,8 +102,8 @@ sq_status sq_check(sq_stream_t stream, uint32_t* device_bits);
  *   Codes and scales are bit-identical to the definition above.  Alignment:
  *   w16, codes 16 B.  A non-finite weight sets SQ_DEV_NONFINITE_WEIGHT.
  * ---------------------------------------------------------------------- */
-size_t sq_quantized_bytes(sq_qkind kind, int64_t N, int64_t K, size_t* scale_bytes);
-sq_status sq_quantize(const void* w16, int64_t N, int64_t K, sq_qkind kind,
+SQ_API size_t sq_quantized_bytes(sq_qkind kind, int64_t N, int64_t K, size_t* scale_bytes);
+SQ_API sq_status sq_quantize(const void* w16, int64_t N, int64_t K, sq_qkind kind,
                       void* codes, void* scales, sq_stream_t stream);
 
 /* ------------------------------------------------------------------------
@@ -111,13 +119,13 @@ sq_status sq_quantize(const void* w16, int64_t N, int64_t K, sq_qkind kind,
  * M runs on the tcgen05 tensor-core tile path where this build has it.
  * y must not overlap x, the weights or the scales.
  * ---------------------------------------------------------------------- */
-sq_status sq_linear_w4a16(const void* x, const void* codes, const void* scales,
+SQ_API sq_status sq_linear_w4a16(const void* x, const void* codes, const void* scales,
                           const void* bias, void* y, int M, int64_t N, int64_t K,
                           sq_stream_t stream);
-sq_status sq_linear_fp8(const void* x, const void* codes, const float* scales,
+SQ_API sq_status sq_linear_fp8(const void* x, const void* codes, const float* scales,
                         const void* bias, void* y, int M, int64_t N, int64_t K,
                         sq_stream_t stream);
-sq_status sq_verify(const void* x, const void* w16, const void* bias, void* y,
+SQ_API sq_status sq_verify(const void* x, const void* w16, const void* bias, void* y,
                     int M, int64_t N, int64_t K, sq_stream_t stream);
 
 /* Fused epilogues of the same three linear layers (the transformer block's
@@ -134,7 +142,7 @@ typedef enum { SQ_W_FP16 = 0, SQ_W_INT4 = 1, SQ_W_FP8 = 2 } sq_wkind;
 /* Generic form of the three linear calls: wkind selects the weight format
  * (w = w16 for SQ_W_FP16, codes otherwise; scales NULL for SQ_W_FP16),
  * epi the epilogue.  residual is read only for SQ_EPI_RESIDUAL. */
-sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void* scales,
+SQ_API sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void* scales,
                        const void* bias, const void* residual, sq_epilogue epi, void* y,
                        int M, int64_t N, int64_t K, sq_stream_t stream);
 
@@ -177,8 +185,8 @@ sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void*
  * call leaves it zero-filled when it completes.  Calls that share one
  * workspace must not run concurrently on the GPU.
  * ---------------------------------------------------------------------- */
-size_t sq_accept_workspace_bytes(int B, int K, int64_t V);
-sq_status sq_accept(const float* p, const float* q, const int32_t* draft, const float* u,
+SQ_API size_t sq_accept_workspace_bytes(int B, int K, int64_t V);
+SQ_API sq_status sq_accept(const float* p, const float* q, const int32_t* draft, const float* u,
                     int B, int K, int64_t V, sq_accept_mode mode,
                     int32_t* n_accepted, int32_t* tokens,
                     void* workspace, size_t ws_bytes, sq_stream_t stream);
@@ -186,7 +194,7 @@ sq_status sq_accept(const float* p, const float* q, const int32_t* draft, const 
 /* Draft-side sampling, token[b] ~ probs[b, :] with uniform u[b]: the K = 0
  * case of sq_accept in sampling mode (same fixed-point inverse CDF, same
  * workspace rules, workspace size sq_accept_workspace_bytes(B, 0, V)). */
-sq_status sq_sample(const float* probs, const float* u, int B, int64_t V, int32_t* tokens,
+SQ_API sq_status sq_sample(const float* probs, const float* u, int B, int64_t V, int32_t* tokens,
                     void* workspace, size_t ws_bytes, sq_stream_t stream);
 
 #ifdef __cplusplus

@@ -3,6 +3,7 @@
 // the hot path; it only checks arguments and launches.
 #include <stdarg.h>
 #include <stdio.h>
+#include <stdlib.h>
 
 #include <string>
 
@@ -39,6 +40,14 @@ int device_sm_count() {
     cache[dev] = n;
   }
   return cache[dev];
+}
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* e = getenv("SQ_PDL");
+    return !(e && e[0] == '0');
+  }();
+  return on;
 }
 
 static int device_max_smem() {
@@ -91,7 +100,6 @@ cudaError_t launch_gemv(int wk, const GemvArgs& a0, cudaStream_t st) {
   GemvArgs a = a0;
   const int cap = gemv_cap_mr(wk, a.K);
   if (cap == 0) return cudaErrorInvalidValue;
-  const int sms = device_sm_count();
   // Rows of x are processed in chunks of at most `cap` (each chunk reads the
   // weights once); M <= 16 with K up to ~19k fits in one or two chunks.
   for (int m0 = 0; m0 < a0.M;) {
@@ -112,15 +120,10 @@ cudaError_t launch_gemv(int wk, const GemvArgs& a0, cudaStream_t st) {
     const int64_t ntiles = (a.N + r - 1) / r;
     const int64_t blocks = (ntiles + 7) / 8;
     const size_t smem = gemv_smem_bytes(wk, mr, a.K);
-    int per_sm = (int)((size_t)(device_max_smem()) / (smem + 1024));
-    if (per_sm > 8) per_sm = 8;
-    if (per_sm < 1) per_sm = 1;
-    const int64_t cap_blocks = (int64_t)sms * per_sm;
-    const int grid = (int)(blocks < cap_blocks ? blocks : cap_blocks);
     cudaError_t e;
-    if (wk == SQ_W_INT4) e = launch_gemv_int4(a, mr, r, silu, grid, smem, st);
-    else if (wk == SQ_W_FP8) e = launch_gemv_fp8(a, mr, r, silu, grid, smem, st);
-    else e = launch_gemv_fp16(a, mr, r, silu, grid, smem, st);
+    if (wk == SQ_W_INT4) e = launch_gemv_int4(a, mr, r, silu, blocks, smem, st);
+    else if (wk == SQ_W_FP8) e = launch_gemv_fp8(a, mr, r, silu, blocks, smem, st);
+    else e = launch_gemv_fp16(a, mr, r, silu, blocks, smem, st);
     if (e != cudaSuccess) return e;
     m0 += m_here;
   }

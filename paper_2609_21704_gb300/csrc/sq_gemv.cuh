@@ -18,9 +18,11 @@
 //     applied once per 32-weight piece; the FP8 row scale once per output;
 //   * the per-lane partial sums are reduced with warp shuffles in a fixed
 //     order, so results are reproducible run to run.
-// Before waiting on the kernel that produces x, each CTA asks L2 to
-// prefetch the first weight bytes it will read (weights never depend on
-// the previous kernel), which overlaps the launch gap with HBM traffic.
+// Each lane keeps U 16-byte pieces of each of its rows in flight per batch
+// (U x 512 B per row per warp), and a warp issues its first batch before
+// waiting on the kernel that produces x: weights never depend on it, so
+// with programmatic dependent launch the weight fetch overlaps that
+// kernel's tail.
 #pragma once
 
 #include "sq_internal.h"
@@ -79,6 +81,14 @@ __device__ __forceinline__ float dot8_natural(uint32_t w0, uint32_t w1, uint32_t
   return acc;
 }
 
+// Pieces of one weight row a lane keeps in flight per batch: enough bytes
+// in flight to cover DRAM latency (U x 512 B per row per warp) within the
+// register budget.
+template <int WR>
+struct Unroll {
+  static constexpr int value = WR == 1 ? 8 : WR == 2 ? 4 : 2;
+};
+
 // MR: activation rows compiled for (M <= MR, missing rows read zeros);
 // R: output rows per warp; SILU: fused gate/up epilogue.
 template <int WK, int MR, int R, bool SILU>
@@ -86,28 +96,48 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
   using T = WTraits<WK>;
   constexpr int SUB = T::kSub;
   constexpr int WR = SILU ? 2 * R : R;  // weight rows per warp tile
+  constexpr int U = Unroll<WR>::value;
   extern __shared__ uint4 xs[];
 
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t ntiles = (a.N + R - 1) / R;
   const int64_t gwarp = (int64_t)blockIdx.x * kGemvWarps + warp;
   const int64_t nwarps = (int64_t)gridDim.x * kGemvWarps;
+  const int steps = a.ppad / 32;
+  const int64_t G = a.K / 128;
 
   auto wrow_index = [&](int64_t tile, int r) -> int64_t {
     if (!SILU) return tile * R + r;
     return r < R ? tile * R + r : a.N + tile * R + (r - R);
   };
   auto row_valid = [&](int64_t tile, int r) -> bool {
-    return tile * R + (SILU ? (r % R) : r) < a.N;
+    return tile < ntiles && tile * R + (SILU ? (r % R) : r) < a.N;
   };
 
-  // L2 prefetch of this warp's first tile (weights do not depend on the
-  // previous kernel, so this overlaps its tail).
-  if (gwarp < ntiles && lane < WR && row_valid(gwarp, lane)) {
-    const uint8_t* row = a.w + wrow_index(gwarp, lane) * a.row_bytes;
-    const int64_t nb = a.row_bytes < 4096 ? a.row_bytes : 4096;
-    prefetch_l2_bulk(row, (uint32_t)(nb & ~15ll));
-  }
+  // One batch = U pieces (steps jb .. jb+U-1) of each of the WR rows.
+  uint4 wv[U][WR];
+  float sv[U][WR];  // INT4 group scales of those pieces
+  auto load_batch = [&](int64_t tile, int jb) {
+#pragma unroll
+    for (int r = 0; r < WR; ++r) {
+      const bool ok = row_valid(tile, r);
+      const int64_t wi = ok ? wrow_index(tile, r) : 0;
+      const uint8_t* row = a.w + wi * a.row_bytes;
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int p = (jb + u) * 32 + lane;
+        const bool in = ok && p < a.pieces;
+        wv[u][r] = in ? ld_stream16(row + (int64_t)p * 16) : make_uint4(0u, 0u, 0u, 0u);
+        if constexpr (WK == WK_INT4)
+          sv[u][r] = in ? __half2float(reinterpret_cast<const __half*>(a.scales)[wi * G + (p >> 2)])
+                        : 0.0f;
+      }
+    }
+  };
+
+  // The weights never depend on the previous kernel: fetch this warp's first
+  // batch before waiting for it.
+  if (gwarp < ntiles) load_batch(gwarp, 0);
 
   griddep_wait();
   griddep_launch_dependents();
@@ -127,89 +157,82 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
   }
   __syncthreads();
 
-  const int steps = a.ppad / 32;
   for (int64_t tile = gwarp; tile < ntiles; tile += nwarps) {
-    const uint8_t* wrow[WR];
-    bool valid[WR];
-#pragma unroll
-    for (int r = 0; r < WR; ++r) {
-      valid[r] = row_valid(tile, r);
-      wrow[r] = a.w + (valid[r] ? wrow_index(tile, r) : 0) * a.row_bytes;
-    }
     float acc[WR][MR];
 #pragma unroll
     for (int r = 0; r < WR; ++r)
 #pragma unroll
       for (int m = 0; m < MR; ++m) acc[r][m] = 0.0f;
 
-    for (int j = 0; j < steps; ++j) {
-      const int p = j * 32 + lane;
-      if (p >= a.pieces) break;
-      uint4 wv[WR];
+    for (int jb = 0; jb < steps; jb += U) {
+      if (jb > 0) load_batch(tile, jb);
 #pragma unroll
-      for (int r = 0; r < WR; ++r)
-        wv[r] = valid[r] ? ld_stream16(wrow[r] + (int64_t)p * 16) : make_uint4(0u, 0u, 0u, 0u);
-
-      if constexpr (WK == WK_INT4) {
-        const __half* sc = reinterpret_cast<const __half*>(a.scales);
-        const int64_t G = a.K / 128;
-        float part[WR][MR];
-#pragma unroll
-        for (int r = 0; r < WR; ++r)
-#pragma unroll
-          for (int m = 0; m < MR; ++m) part[r][m] = 0.0f;
-#pragma unroll
-        for (int i = 0; i < SUB; ++i) {
-          uint32_t c[WR][4];
-#pragma unroll
-          for (int r = 0; r < WR; ++r) {
-            const uint32_t word = i == 0 ? wv[r].x : i == 1 ? wv[r].y : i == 2 ? wv[r].z : wv[r].w;
-            int4x8_to_f16x2(word, c[r]);
-          }
-#pragma unroll
-          for (int m = 0; m < MR; ++m) {
-            const uint4 xq = xs[m * chunks_per_m + (j * SUB + i) * 32 + lane];
-#pragma unroll
-            for (int r = 0; r < WR; ++r) part[r][m] = dot8_int4order(c[r], xq, part[r][m]);
-          }
-        }
-#pragma unroll
-        for (int r = 0; r < WR; ++r) {
-          const float s = valid[r] ? __half2float(sc[wrow_index(tile, r) * G + (p >> 2)]) : 0.0f;
-#pragma unroll
-          for (int m = 0; m < MR; ++m) acc[r][m] = fmaf(s, part[r][m], acc[r][m]);
-        }
-      } else if constexpr (WK == WK_FP8) {
-#pragma unroll
-        for (int i = 0; i < SUB; ++i) {
-          uint32_t h[WR][4];
-#pragma unroll
-          for (int r = 0; r < WR; ++r) {
-            const uint32_t wa = i == 0 ? wv[r].x : wv[r].z;
-            const uint32_t wb = i == 0 ? wv[r].y : wv[r].w;
-            h[r][0] = e4m3x2_to_f16x2(lo16(wa));
-            h[r][1] = e4m3x2_to_f16x2(hi16(wa));
-            h[r][2] = e4m3x2_to_f16x2(lo16(wb));
-            h[r][3] = e4m3x2_to_f16x2(hi16(wb));
-          }
-#pragma unroll
-          for (int m = 0; m < MR; ++m) {
-            const uint4 xq = xs[m * chunks_per_m + (j * SUB + i) * 32 + lane];
-#pragma unroll
-            for (int r = 0; r < WR; ++r)
-              acc[r][m] = dot8_natural(h[r][0], h[r][1], h[r][2], h[r][3], xq, acc[r][m]);
-          }
-        }
-      } else {
-#pragma unroll
-        for (int m = 0; m < MR; ++m) {
-          const uint4 xq = xs[m * chunks_per_m + j * 32 + lane];
+      for (int u = 0; u < U; ++u) {
+        const int j = jb + u;
+        if (j * 32 >= a.pieces) break;  // warp-uniform
+        if constexpr (WK == WK_INT4) {
+          float part[WR][MR];
 #pragma unroll
           for (int r = 0; r < WR; ++r)
-            acc[r][m] = dot8_natural(wv[r].x, wv[r].y, wv[r].z, wv[r].w, xq, acc[r][m]);
+#pragma unroll
+            for (int m = 0; m < MR; ++m) part[r][m] = 0.0f;
+#pragma unroll
+          for (int i = 0; i < SUB; ++i) {
+            uint32_t c[WR][4];
+#pragma unroll
+            for (int r = 0; r < WR; ++r) {
+              const uint4 w = wv[u][r];
+              const uint32_t word = i == 0 ? w.x : i == 1 ? w.y : i == 2 ? w.z : w.w;
+              int4x8_to_f16x2(word, c[r]);
+            }
+#pragma unroll
+            for (int m = 0; m < MR; ++m) {
+              const uint4 xq = xs[m * chunks_per_m + (j * SUB + i) * 32 + lane];
+#pragma unroll
+              for (int r = 0; r < WR; ++r) part[r][m] = dot8_int4order(c[r], xq, part[r][m]);
+            }
+          }
+#pragma unroll
+          for (int r = 0; r < WR; ++r)
+#pragma unroll
+            for (int m = 0; m < MR; ++m) acc[r][m] = fmaf(sv[u][r], part[r][m], acc[r][m]);
+        } else if constexpr (WK == WK_FP8) {
+#pragma unroll
+          for (int i = 0; i < SUB; ++i) {
+            uint32_t h[WR][4];
+#pragma unroll
+            for (int r = 0; r < WR; ++r) {
+              const uint4 w = wv[u][r];
+              const uint32_t wa = i == 0 ? w.x : w.z;
+              const uint32_t wb = i == 0 ? w.y : w.w;
+              h[r][0] = e4m3x2_to_f16x2(lo16(wa));
+              h[r][1] = e4m3x2_to_f16x2(hi16(wa));
+              h[r][2] = e4m3x2_to_f16x2(lo16(wb));
+              h[r][3] = e4m3x2_to_f16x2(hi16(wb));
+            }
+#pragma unroll
+            for (int m = 0; m < MR; ++m) {
+              const uint4 xq = xs[m * chunks_per_m + (j * SUB + i) * 32 + lane];
+#pragma unroll
+              for (int r = 0; r < WR; ++r)
+                acc[r][m] = dot8_natural(h[r][0], h[r][1], h[r][2], h[r][3], xq, acc[r][m]);
+            }
+          }
+        } else {
+#pragma unroll
+          for (int m = 0; m < MR; ++m) {
+            const uint4 xq = xs[m * chunks_per_m + j * 32 + lane];
+#pragma unroll
+            for (int r = 0; r < WR; ++r) {
+              const uint4 w = wv[u][r];
+              acc[r][m] = dot8_natural(w.x, w.y, w.z, w.w, xq, acc[r][m]);
+            }
+          }
         }
       }
     }
+    // prefetch the next tile's first batch before the reduction
+    if (tile + nwarps < ntiles) load_batch(tile + nwarps, 0);
 
     // ---- reduce across the warp (fixed butterfly order)
 #pragma unroll
@@ -241,29 +264,55 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
   }
 }
 
-// Instantiation helper used by the per-format translation units.
+// Instantiation helper used by the per-format translation units.  The grid
+// is persistent: at most as many CTAs as can be resident at once (from the
+// occupancy calculator), each warp looping over tiles.
 template <int WK, int MR, int R, bool SILU>
-cudaError_t launch_gemv_inst(const GemvArgs& a, int grid, size_t smem, cudaStream_t st) {
+cudaError_t launch_gemv_inst(const GemvArgs& a, int64_t blocks_needed, size_t smem,
+                             cudaStream_t st) {
   auto k = gemv_kernel<WK, MR, R, SILU>;
-  static int smem_set[64] = {0};  // per device: largest dynamic smem enabled so far
+  struct Cached {
+    int smem_set = 0;
+    size_t occ_smem[8] = {0};
+    int occ[8] = {0};
+  };
+  static Cached cache[64];  // per device
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if (smem > 48 * 1024 && dev < 64 && (int)smem > smem_set[dev]) {
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  Cached& c = cache[dev];
+  if (smem > 48 * 1024 && (int)smem > c.smem_set) {
     e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    smem_set[dev] = (int)smem;
+    c.smem_set = (int)smem;
   }
-  return launch_pdl(k, dim3(grid), dim3(kGemvThreads), smem, st, a);
+  int occ = 0;
+  for (int i = 0; i < 8; ++i)
+    if (c.occ_smem[i] == smem + 1) occ = c.occ[i];
+  if (occ == 0) {
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k, kGemvThreads, smem);
+    if (e != cudaSuccess) return e;
+    if (occ < 1) occ = 1;
+    for (int i = 0; i < 8; ++i)
+      if (c.occ_smem[i] == 0) {
+        c.occ_smem[i] = smem + 1;
+        c.occ[i] = occ;
+        break;
+      }
+  }
+  const int64_t cap = (int64_t)device_sm_count() * occ;
+  const int grid = (int)(blocks_needed < cap ? blocks_needed : cap);
+  return launch_pdl(k, dim3(grid > 0 ? grid : 1), dim3(kGemvThreads), smem, st, a);
 }
 
 template <int WK>
-cudaError_t launch_gemv_fmt(const GemvArgs& a, int mr, int r, bool silu, int grid, size_t smem,
-                            cudaStream_t st) {
+cudaError_t launch_gemv_fmt(const GemvArgs& a, int mr, int r, bool silu, int64_t blocks_needed,
+                            size_t smem, cudaStream_t st) {
 #define SQ_GEMV_CASE(MR_, R_)                                                              \
   if (mr == MR_ && r == R_)                                                                \
-    return silu ? launch_gemv_inst<WK, MR_, R_, true>(a, grid, smem, st)                   \
-                : launch_gemv_inst<WK, MR_, R_, false>(a, grid, smem, st);
+    return silu ? launch_gemv_inst<WK, MR_, R_, true>(a, blocks_needed, smem, st)          \
+                : launch_gemv_inst<WK, MR_, R_, false>(a, blocks_needed, smem, st);
   SQ_GEMV_CASE(1, 1)
   SQ_GEMV_CASE(1, 2)
   SQ_GEMV_CASE(2, 1)

@@ -5,9 +5,9 @@
 
 namespace sq {
 
-cudaError_t launch_gemv_int4(const GemvArgs& a, int mr, int r, bool silu, int grid, size_t smem,
+cudaError_t launch_gemv_int4(const GemvArgs& a, int mr, int r, bool silu, int64_t blocks_needed, size_t smem,
                            cudaStream_t st) {
-  return launch_gemv_fmt<WK_INT4>(a, mr, r, silu, grid, smem, st);
+  return launch_gemv_fmt<WK_INT4>(a, mr, r, silu, blocks_needed, smem, st);
 }
 
 }  // namespace sq

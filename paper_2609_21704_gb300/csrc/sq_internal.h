@@ -12,6 +12,7 @@ namespace sq {
 constexpr int kNumSMs = 152;  // GB300: 2 dies x 76 SMs (queried at run time too)
 
 int device_sm_count();
+bool pdl_enabled();  // SQ_PDL environment knob, read once
 
 // Launch with programmatic dependent launch allowed: the kernel may begin
 // while the previous kernel on the stream drains; it must call
@@ -29,8 +30,9 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   const bool legacy = (st == nullptr || st == cudaStreamLegacy || st == cudaStreamPerThread);
-  cfg.attrs = legacy ? nullptr : attr;
-  cfg.numAttrs = legacy ? 0 : 1;
+  const bool pdl = !legacy && pdl_enabled();
+  cfg.attrs = pdl ? attr : nullptr;
+  cfg.numAttrs = pdl ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
@@ -61,12 +63,14 @@ constexpr int kGemvMaxRows = 16;
 size_t gemv_smem_bytes(int wkind, int mr, int64_t K);
 int gemv_pick_mr(int M);
 cudaError_t launch_gemv(int wkind, const GemvArgs& a, cudaStream_t st);
-cudaError_t launch_gemv_int4(const GemvArgs& a, int mr, int r, bool silu, int grid, size_t smem,
-                             cudaStream_t st);
-cudaError_t launch_gemv_fp8(const GemvArgs& a, int mr, int r, bool silu, int grid, size_t smem,
-                            cudaStream_t st);
-cudaError_t launch_gemv_fp16(const GemvArgs& a, int mr, int r, bool silu, int grid, size_t smem,
-                             cudaStream_t st);
+// blocks_needed: CTAs that would give every warp one tile; the launcher
+// caps it at the number of CTAs that can be resident at once.
+cudaError_t launch_gemv_int4(const GemvArgs& a, int mr, int r, bool silu, int64_t blocks_needed,
+                             size_t smem, cudaStream_t st);
+cudaError_t launch_gemv_fp8(const GemvArgs& a, int mr, int r, bool silu, int64_t blocks_needed,
+                            size_t smem, cudaStream_t st);
+cudaError_t launch_gemv_fp16(const GemvArgs& a, int mr, int r, bool silu, int64_t blocks_needed,
+                             size_t smem, cudaStream_t st);
 
 // sq_accept.cu
 struct AcceptArgs {
