@@ -197,6 +197,35 @@ SQ_API sq_status sq_accept(const float* p, const float* q, const int32_t* draft,
 SQ_API sq_status sq_sample(const float* probs, const float* u, int B, int64_t V, int32_t* tokens,
                     void* workspace, size_t ws_bytes, sq_stream_t stream);
 
+/* ------------------------------------------------------------------------
+ * sq_accept_noalloc: sq_accept without a caller workspace.  The paper has
+ * no counterpart; it exists for callers that cannot allocate device memory
+ * where they run the accept step -- code inside a host framework that owns
+ * every device byte through its own pool and does not let components call
+ * cudaMalloc, or a latency-critical loop where an allocation (which may
+ * synchronise the device) is not acceptable.
+ *
+ * Same arguments, semantics, limits and results as sq_accept, minus the
+ * workspace.  The scratch is a static device array inside the library of
+ * SQ_ACCEPT_NOALLOC_SCRATCH_BYTES (1 MiB); every GPU that loads the library
+ * holds it until the process exits.  A call whose
+ * sq_accept_workspace_bytes(B, K, V) exceeds that size is rejected with
+ * SQ_ERR_SHAPE (e.g. V = 152064 with K = 4 fits up to B = 349).  The call clears
+ * the ticket counters in the scratch on `stream` before launching and never
+ * calls cudaMalloc, cudaFree or any allocating routine.
+ *
+ * Every call on a device shares the one scratch array, which keeps the last
+ * call's contents: calls that overlap on the GPU (two streams, two host
+ * threads) race and give wrong results; serialise them.
+ * The first call on a device looks up the scratch's device address (once per
+ * device, with that device current); make that first call before any stream
+ * capture begins.
+ * ---------------------------------------------------------------------- */
+#define SQ_ACCEPT_NOALLOC_SCRATCH_BYTES ((size_t)1 << 20)
+SQ_API sq_status sq_accept_noalloc(const float* p, const float* q, const int32_t* draft,
+                                   const float* u, int B, int K, int64_t V, sq_accept_mode mode,
+                                   int32_t* n_accepted, int32_t* tokens, sq_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

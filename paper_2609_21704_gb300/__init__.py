@@ -26,7 +26,7 @@ __all__ = [
     "SQ_EPI_NONE", "SQ_EPI_SILU_GATE", "SQ_EPI_RESIDUAL", "SQ_W_FP16", "SQ_W_INT4", "SQ_W_FP8",
     "sq_quantized_bytes", "sq_quantize", "sq_linear_w4a16", "sq_linear_fp8", "sq_verify",
     "sq_linear_ex", "sq_accept_workspace_bytes", "sq_accept", "sq_sample", "sq_check",
-    "sq_version", "EXPORTED_SYMBOLS",
+    "sq_version", "sq_accept_noalloc", "EXPORTED_SYMBOLS",
 ]
 
 SQ_OK = 0
@@ -54,6 +54,7 @@ _SIGS = {
     "sq_accept_workspace_bytes": (_SIZE, [_INT, _INT, _I64]),
     "sq_accept": (_INT, [_P, _P, _P, _P, _INT, _INT, _I64, _INT, _P, _P, _P, _SIZE, _P]),
     "sq_sample": (_INT, [_P, _P, _INT, _I64, _P, _P, _SIZE, _P]),
+    "sq_accept_noalloc": (_INT, [_P, _P, _P, _P, _INT, _INT, _I64, _INT, _P, _P, _P]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGS)
 
@@ -167,6 +168,15 @@ def sq_accept(p, q, draft, u, mode, n_accepted, tokens, workspace, stream=None) 
                                          _ptr(n_accepted), _ptr(tokens), _ptr(workspace),
                                          workspace.numel() * workspace.element_size(),
                                          _stream(stream)))
+
+
+def sq_accept_noalloc(p, q, draft, u, mode, n_accepted, tokens, stream=None) -> None:
+    """sq_accept without a workspace, for callers that cannot allocate
+    device memory: the library's static 1 MiB scratch is used instead."""
+    B, K1, V = p.shape
+    _check("sq_accept_noalloc", load().sq_accept_noalloc(_ptr(p), _ptr(q), _ptr(draft), _ptr(u), B,
+                                                         K1 - 1, V, mode, _ptr(n_accepted),
+                                                         _ptr(tokens), _stream(stream)))
 
 
 def sq_sample(probs, u, tokens, workspace, stream=None) -> None:

@@ -16,11 +16,19 @@
 //
 // Bytes per sequence: sampling 2 V fp32 (p_n and q_n) + 2K gathers;
 // greedy (K+1) V fp32.
+#include <mutex>
+
 #include "sq_internal.h"
 
 namespace sq {
 
 __device__ unsigned int g_accept_status;
+
+// Scratch of sq_accept_noalloc: ticket counters and per-chunk partials live
+// here instead of in a caller-provided workspace.  Every device that loads
+// the library keeps this array until the process exits, and every call of
+// sq_accept_noalloc on a device reuses the same bytes.
+static __device__ __align__(256) unsigned char g_accept_scratch[kAcceptNoallocScratchBytes];
 
 // floor(r * 2^44) from the fp32 bits of r in [0, 1] (exact integer shifts).
 __device__ __forceinline__ unsigned long long fix44(float r) {
@@ -297,6 +305,27 @@ cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t st) {
   if (a.B == 0) return cudaSuccess;
   const int64_t blocks = (int64_t)a.B * a.C;
   return launch_pdl(accept_kernel, dim3((unsigned)blocks), dim3(kAcceptThreads), 0, st, a);
+}
+
+// Device address of g_accept_scratch for the current device.  In host code
+// the array's name is only a host-side stand-in, so the address is asked of
+// the runtime once per device (with that device current) and cached.
+cudaError_t accept_noalloc_scratch(void** ptr) {
+  static std::mutex mu;
+  static void* addr[64] = {nullptr};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (addr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_accept_scratch);
+    if (e != cudaSuccess) return e;
+    addr[dev] = p;
+  }
+  *ptr = addr[dev];
+  return cudaSuccess;
 }
 
 cudaError_t take_accept_status(uint32_t* bits) {

@@ -328,4 +328,32 @@ sq_status sq_sample(const float* probs, const float* u, int B, int64_t V, int32_
                        tokens, workspace, ws_bytes, stream);
 }
 
+// Same step as sq_accept for callers that cannot allocate device memory:
+// the scratch is the library's own static device array (see sq_accept.cu).
+// The ticket counters in it are cleared on the stream before each launch;
+// nothing here allocates.
+sq_status sq_accept_noalloc(const float* p, const float* q, const int32_t* draft, const float* u,
+                            int B, int K, int64_t V, sq_accept_mode mode, int32_t* n_accepted,
+                            int32_t* tokens, sq_stream_t stream) {
+  if (B < 0 || K < 0 || K > 16 || V < 1 || V >= ((int64_t)1 << 20))
+    return fail(SQ_ERR_SHAPE, "sq_accept_noalloc: need B >= 0, 0 <= K <= 16, 1 <= V < 2^20 (B=%d K=%d V=%lld)",
+                B, K, (long long)V);
+  if (B == 0) return SQ_OK;
+  if (!n_accepted) return fail(SQ_ERR_INVALID_ARG, "sq_accept_noalloc: NULL n_accepted");
+  const size_t need = accept_workspace_bytes(B, K, V);
+  if (need > kAcceptNoallocScratchBytes)
+    return fail(SQ_ERR_SHAPE,
+                "sq_accept_noalloc: B=%d K=%d V=%lld needs %zu bytes of scratch but the static scratch "
+                "holds %zu; use sq_accept with a workspace, or fewer sequences per call",
+                B, K, (long long)V, need, kAcceptNoallocScratchBytes);
+  void* scratch = nullptr;
+  cudaError_t e = accept_noalloc_scratch(&scratch);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_accept_noalloc: scratch address");
+  const size_t ctr = (((size_t)B * 4u) + 15u) & ~(size_t)15u;
+  e = cudaMemsetAsync(scratch, 0, ctr, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_accept_noalloc: clearing the ticket counters");
+  return accept_common("sq_accept_noalloc", p, q, draft, u, B, K, V, (int)mode, n_accepted, tokens,
+                       scratch, kAcceptNoallocScratchBytes, stream);
+}
+
 }  // extern "C"

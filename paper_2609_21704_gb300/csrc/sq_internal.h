@@ -91,6 +91,9 @@ struct AcceptArgs {
 };
 constexpr int kAcceptChunk = 2048;
 size_t accept_workspace_bytes(int B, int K, int64_t V);
+// Size of the static scratch behind sq_accept_noalloc (1 MiB).
+constexpr size_t kAcceptNoallocScratchBytes = (size_t)1 << 20;
+cudaError_t accept_noalloc_scratch(void** ptr);
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t st);
 cudaError_t take_accept_status(uint32_t* bits);
 
