@@ -52,6 +52,12 @@ def parse():
     ap.add_argument("--batch", type=int, default=1, help="sequences per GPU")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="decoder layers to build (default: the workload's; --case runs only)")
+    ap.add_argument("--case", default=None,
+                    help="time one kernel class over all layers instead of the step (for ncu): "
+                         "draft_qkv|draft_o|draft_gateup|draft_down|draft_lm|verify_qkv|verify_o|"
+                         "verify_gateup|verify_down|verify_lm|accept")
     return ap.parse_args()
 
 
@@ -141,14 +147,24 @@ def barrier(world):
 
 
 def max_over_ranks(x, world):
+    """Largest value of x over the ranks (the timed region of the slowest
+    replica); a CPU tensor under gloo, a device tensor under nccl."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
 
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def aggregate_tokens_per_s(tokens_per_step_per_rank, steps, t_max, world):
+    """Whole-job throughput of independent replicas: every rank emits
+    tokens_per_step_per_rank tokens per step; the job takes as long as its
+    slowest rank."""
+    return world * tokens_per_step_per_rank * steps / t_max
 
 
 def source_digest(paths):
@@ -259,7 +275,10 @@ def main():
 
     # ---- one GPU replica: weights, variants, buffers
     t0 = time.perf_counter()
-    stack = stk.LinearStack(shape, dev, seed=1000 * rank, variants=("int4", "fp8"))
+    if args.layers is not None and not args.case:
+        raise SystemExit("--layers is only for --case runs; the step always uses the whole stack")
+    variants = ("int4", "fp8") if not args.case else ((args.draft,) if args.case.startswith("draft") else ())
+    stack = stk.LinearStack(shape, dev, seed=1000 * rank, variants=variants, layers=args.layers)
     torch.cuda.synchronize()
     derive_s = time.perf_counter() - t0
     bd = stk.PassBuffers(stack, B, seed=11 + rank)
@@ -283,6 +302,8 @@ def main():
     alpha = float(n_cal.float().mean().item()) / K
 
     stream = torch.cuda.Stream(device=dev)
+    if args.case:
+        return run_case(args, stack, bd, bv, (tp, tq, td, tu, n_out, tok_out, ws), stream, peak_gbs)
 
     def step():
         for _ in range(K):
@@ -331,7 +352,7 @@ def main():
     t_step = max_over_ranks(t_step, world)
     ms_per_step = 1e3 * t_step / args.steps
     tokens_per_step = B * mean_tokens
-    value = world * tokens_per_step * args.steps / t_step
+    value = aggregate_tokens_per_s(tokens_per_step, args.steps, t_step, world)
 
     # ---- breakdown: each pass type alone (graphs), algorithmic bytes / time
     def pass_graph(variant, bufs):
@@ -410,7 +431,7 @@ def main():
         for _ in range(e2e_steps):
             e2e_step()
         t_e2e = max_over_ranks(time.perf_counter() - t0, world)
-        e2e = {"value": world * tokens_per_step * e2e_steps / t_e2e, "unit": UNIT,
+        e2e = {"value": aggregate_tokens_per_s(tokens_per_step, e2e_steps, t_e2e, world), "unit": UNIT,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                "ms_per_step": 1e3 * t_e2e / e2e_steps, "steps": e2e_steps}
 
@@ -465,6 +486,53 @@ def main():
         "gpu_launches": launches_per_step * args.steps,
     }
     print(json.dumps(out))
+    return 0
+
+
+def run_case(args, stack, bd, bv, acc, stream, peak_gbs):
+    """One kernel class over all layers, eagerly (no graph), `--warmup` then
+    `--steps` iterations timed with CUDA events; prints one JSON line."""
+    import torch
+
+    import paper_2609_21704_gb300 as sq
+    from paper_2609_21704_gb300 import stack as stk
+
+    side, _, what = args.case.partition("_")
+    if args.case == "accept":
+        tp, tq, td, tu, n_out, tok_out, ws = acc
+
+        def once():
+            sq.sq_accept(tp, tq, td, tu, sq.SQ_ACCEPT_SAMPLE, n_out, tok_out, ws, stream)
+        nbytes, launches = tp.shape[0] * (2 * tp.shape[2] * 4), 1
+    else:
+        variant = args.draft if side == "draft" else "fp16"
+        bufs = bd if side == "draft" else bv
+        idx = {"qkv": 0, "o": 1, "gateup": 2, "down": 3}.get(what)
+        projs = [stack.lm_head] if what == "lm" else [layer[idx] for layer in stack.layers]
+        ins = {"qkv": bufs.x, "o": bufs.attn, "gateup": bufs.x, "down": bufs.h, "lm": bufs.x}[what]
+        outs = {"qkv": bufs.qkv, "o": bufs.o, "gateup": bufs.h, "down": bufs.d, "lm": bufs.logits}[what]
+        wk = stk.WKIND[variant]
+
+        def once():
+            for pr in projs:
+                w, s = pr.weight(variant)
+                sq.sq_linear_ex(wk, ins, w, s, None, None, pr.epi, outs, stream)
+        nbytes = sum(pr.weight_bytes(variant) + 2 * bufs.M * (pr.k_in + pr.y_cols()) for pr in projs)
+        launches = len(projs)
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            once()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            once()
+        e1.record(stream)
+    e1.synchronize()
+    t = e0.elapsed_time(e1) / 1e3 / args.steps
+    print(json.dumps({"case": args.case, "launches_per_iter": launches, "us_per_launch": 1e6 * t / launches,
+                      "bytes_per_launch": nbytes / launches, "gbs": nbytes / t / 1e9,
+                      "frac_of_peak": nbytes / t / 1e9 / peak_gbs, "eager": True}))
     return 0
 
 
