@@ -15,9 +15,14 @@
  *    the call returns.  Row-major, densely packed, no strides.
  *  - Every call is asynchronous and ordered on `stream` (NULL = the legacy
  *    default stream).  Kernels are launched with programmatic dependent
- *    launch allowed, so a call may start fetching its weights while the
- *    previous kernel on the stream finishes; it reads activations and writes
- *    outputs only after that kernel completed.
+ *    launch allowed, so a linear call may start fetching its weights while
+ *    the previous kernel on the stream finishes; it reads activations and
+ *    writes outputs only after that kernel completed.  Consequence: the
+ *    weights and scales of a linear call must not be written by the call
+ *    issued immediately before it on the same stream if that call is a
+ *    linear or accept call of this library (those let the next kernel start
+ *    early).  Writes by sq_quantize, by copies and by other libraries'
+ *    kernels are always complete first.
  *  - Return value: SQ_OK, or an error code whose text sq_last_error()
  *    returns (per host thread).  Arguments are validated on the host before
  *    anything is launched; an invalid call launches nothing.  No call traps,
@@ -68,6 +73,7 @@ typedef enum { SQ_ACCEPT_SAMPLE = 0, SQ_ACCEPT_GREEDY = 1 } sq_accept_mode;
 #define SQ_DEV_BAD_DRAFT_TOKEN  0x2u  /* sq_accept: draft token not in [0,V) */
 #define SQ_DEV_NO_MASS          0x4u  /* sq_accept/sq_sample: row w/o mass   */
 #define SQ_DEV_BAD_UNIFORM      0x8u  /* resampling uniform not in [0,1)     */
+#define SQ_DEV_TIMEOUT          0x10u /* a kernel gave up a bounded wait     */
 
 /* Thread-local text of the last error raised on this host thread. */
 SQ_API const char* sq_last_error(void);

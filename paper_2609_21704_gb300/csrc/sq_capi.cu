@@ -160,6 +160,10 @@ sq_status sq_check(sq_stream_t stream, uint32_t* device_bits) {
   uint32_t bits = 0;
   if ((e = take_quant_status(&bits)) != cudaSuccess) return cuda_fail(e, "sq_check: quantize status");
   if ((e = take_accept_status(&bits)) != cudaSuccess) return cuda_fail(e, "sq_check: accept status");
+  if ((e = take_gemv_status_int4(&bits)) != cudaSuccess ||
+      (e = take_gemv_status_fp8(&bits)) != cudaSuccess ||
+      (e = take_gemv_status_fp16(&bits)) != cudaSuccess)
+    return cuda_fail(e, "sq_check: linear status");
   if (device_bits) *device_bits = bits;
   if (bits) return fail(SQ_ERR_DEVICE, "sq_check: device status bits 0x%x", bits);
   return SQ_OK;

@@ -18,11 +18,16 @@
 //     applied once per 32-weight piece; the FP8 row scale once per output;
 //   * the per-lane partial sums are reduced with warp shuffles in a fixed
 //     order, so results are reproducible run to run.
-// Each lane keeps U 16-byte pieces of each of its rows in flight per batch
-// (U x 512 B per row per warp), and a warp issues its first batch before
-// waiting on the kernel that produces x: weights never depend on it, so
-// with programmatic dependent launch the weight fetch overlaps that
-// kernel's tail.
+// Each CTA owns a contiguous slice of row tiles and each warp the tiles
+// w, w + 8, ... of it.  A lane keeps U 16-byte pieces of each of its rows in
+// flight per batch (U x 512 B per row per warp), and every warp keeps the
+// bytes of its next kPrefetchTiles tiles requested into L2 with bulk
+// prefetches (cp.async.bulk.prefetch.L2).  The first batch and the first
+// prefetches are issued before waiting on the kernel that produces x:
+// weights never depend on it, so with programmatic dependent launch the
+// weight fetch overlaps that kernel's tail.  The grid holds as many CTAs as
+// can be resident at once (occupancy calculator): many warps per SM are
+// what keeps the issue slots busy.
 #pragma once
 
 #include "sq_internal.h"
@@ -51,6 +56,10 @@ struct WTraits<WK_FP16> {
 
 constexpr int kGemvThreads = 256;
 constexpr int kGemvWarps = kGemvThreads / 32;
+constexpr int kPrefetchTiles = 2;  // tiles of its own a warp keeps requested into L2
+
+// Status word of the GEMV kernels of one translation unit.
+static __device__ unsigned int g_gemv_status;
 
 // acc[m] += sum_{j<8} c_j * x_j for one 8-weight chunk; c holds the codes as
 // fp16 pairs (c0,c4),(c1,c5),(c2,c6),(c3,c7) (INT4 order) and xq the chunk
@@ -101,8 +110,11 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
 
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t ntiles = (a.N + R - 1) / R;
-  const int64_t gwarp = (int64_t)blockIdx.x * kGemvWarps + warp;
-  const int64_t nwarps = (int64_t)gridDim.x * kGemvWarps;
+  // this CTA's slice of tiles [t_begin, t_end); warp w takes t_begin + w + 8 i
+  const int64_t t_begin = ((int64_t)blockIdx.x * ntiles) / gridDim.x;
+  const int64_t t_end = ((int64_t)(blockIdx.x + 1) * ntiles) / gridDim.x;
+  const int64_t gwarp = t_begin + warp;
+  const int64_t nwarps = kGemvWarps;
   const int steps = a.ppad / 32;
   const int64_t G = a.K / 128;
 
@@ -111,7 +123,17 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
     return r < R ? tile * R + r : a.N + tile * R + (r - R);
   };
   auto row_valid = [&](int64_t tile, int r) -> bool {
-    return tile < ntiles && tile * R + (SILU ? (r % R) : r) < a.N;
+    return tile < t_end && tile * R + (SILU ? (r % R) : r) < a.N;
+  };
+  // L2 bulk prefetch of one tile's rows (lane r < WR takes row r).
+  auto prefetch_tile = [&](int64_t tile) {
+    if (lane < WR && row_valid(tile, lane)) {
+      const uint8_t* row = a.w + wrow_index(tile, lane) * a.row_bytes;
+      for (int64_t off = 0; off < a.row_bytes; off += 32768) {
+        const int64_t nb = a.row_bytes - off < 32768 ? a.row_bytes - off : 32768;
+        prefetch_l2_bulk(row + off, (uint32_t)nb);
+      }
+    }
   };
 
   // One batch = U pieces (steps jb .. jb+U-1) of each of the WR rows.
@@ -135,9 +157,11 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
     }
   };
 
-  // The weights never depend on the previous kernel: fetch this warp's first
-  // batch before waiting for it.
-  if (gwarp < ntiles) load_batch(gwarp, 0);
+  // The weights never depend on the previous kernel: request this warp's
+  // next tiles into L2 and fetch its first batch before waiting for it.
+#pragma unroll
+  for (int d = 1; d <= kPrefetchTiles; ++d) prefetch_tile(gwarp + (int64_t)d * nwarps);
+  if (gwarp < t_end) load_batch(gwarp, 0);
 
   griddep_wait();
   griddep_launch_dependents();
@@ -157,7 +181,8 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
   }
   __syncthreads();
 
-  for (int64_t tile = gwarp; tile < ntiles; tile += nwarps) {
+  for (int64_t tile = gwarp; tile < t_end; tile += nwarps) {
+    prefetch_tile(tile + (int64_t)(kPrefetchTiles + 1) * nwarps);
     float acc[WR][MR];
 #pragma unroll
     for (int r = 0; r < WR; ++r)
@@ -232,7 +257,7 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
       }
     }
     // prefetch the next tile's first batch before the reduction
-    if (tile + nwarps < ntiles) load_batch(tile + nwarps, 0);
+    if (tile + nwarps < t_end) load_batch(tile + nwarps, 0);
 
     // ---- reduce across the warp (fixed butterfly order)
 #pragma unroll
@@ -265,8 +290,8 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
 }
 
 // Instantiation helper used by the per-format translation units.  The grid
-// is persistent: at most as many CTAs as can be resident at once (from the
-// occupancy calculator), each warp looping over tiles.
+// is persistent: at most as many CTAs as can be resident at once, each warp
+// looping over the tiles of its CTA's slice.
 template <int WK, int MR, int R, bool SILU>
 cudaError_t launch_gemv_inst(const GemvArgs& a, int64_t blocks_needed, size_t smem,
                              cudaStream_t st) {
@@ -325,6 +350,16 @@ cudaError_t launch_gemv_fmt(const GemvArgs& a, int mr, int r, bool silu, int64_t
   SQ_GEMV_CASE(16, 1)
 #undef SQ_GEMV_CASE
   return cudaErrorInvalidValue;
+}
+
+// Reads and clears this translation unit's status word.
+inline cudaError_t take_gemv_status_tu(uint32_t* bits) {
+  uint32_t v = 0, zero = 0;
+  cudaError_t e = cudaMemcpyFromSymbol(&v, g_gemv_status, sizeof(v));
+  if (e != cudaSuccess) return e;
+  if (v) e = cudaMemcpyToSymbol(g_gemv_status, &zero, sizeof(zero));
+  *bits |= v;
+  return e;
 }
 
 }  // namespace sq

@@ -10,4 +10,6 @@ cudaError_t launch_gemv_fp16(const GemvArgs& a, int mr, int r, bool silu, int64_
   return launch_gemv_fmt<WK_FP16>(a, mr, r, silu, blocks_needed, smem, st);
 }
 
+cudaError_t take_gemv_status_fp16(uint32_t* bits) { return take_gemv_status_tu(bits); }
+
 }  // namespace sq

@@ -10,4 +10,6 @@ cudaError_t launch_gemv_fp8(const GemvArgs& a, int mr, int r, bool silu, int64_t
   return launch_gemv_fmt<WK_FP8>(a, mr, r, silu, blocks_needed, smem, st);
 }
 
+cudaError_t take_gemv_status_fp8(uint32_t* bits) { return take_gemv_status_tu(bits); }
+
 }  // namespace sq

@@ -71,6 +71,9 @@ cudaError_t launch_gemv_fp8(const GemvArgs& a, int mr, int r, bool silu, int64_t
                             size_t smem, cudaStream_t st);
 cudaError_t launch_gemv_fp16(const GemvArgs& a, int mr, int r, bool silu, int64_t blocks_needed,
                              size_t smem, cudaStream_t st);
+cudaError_t take_gemv_status_int4(uint32_t* bits);
+cudaError_t take_gemv_status_fp8(uint32_t* bits);
+cudaError_t take_gemv_status_fp16(uint32_t* bits);
 
 // sq_accept.cu
 struct AcceptArgs {

@@ -7,6 +7,9 @@
 //   FP8:  per output row, s = fp32(amax / 448), code = E4M3_satfinite(w / s).
 // Every division is the IEEE fp32 divide (__fdiv_rn) and every rounding is
 // to nearest even, so codes and scales are bit-identical to the definition.
+// These kernels never let the next kernel start early: linear kernels read
+// their weights before waiting on the previous kernel, and the weights may
+// be what this kernel writes.
 // Both kernels are HBM-bound streaming passes: 2 B read per weight, 0.516 B
 // (INT4) or 1 B (FP8) written.
 #include "sq_internal.h"
@@ -19,8 +22,7 @@ __device__ unsigned int g_quant_status;
 __global__ void __launch_bounds__(256) quant_int4_kernel(const __half* __restrict__ w, int64_t N,
                                                          int64_t K, uint8_t* __restrict__ codes,
                                                          __half* __restrict__ scales) {
-  griddep_wait();
-  griddep_launch_dependents();
+  griddep_wait();  // no early trigger: a linear call may read these outputs at once
   const int lane = threadIdx.x & 31;
   const int64_t G = K / 128;
   const int64_t total = N * G;
@@ -68,8 +70,7 @@ __global__ void __launch_bounds__(256) quant_int4_kernel(const __half* __restric
 __global__ void __launch_bounds__(256) quant_fp8_kernel(const __half* __restrict__ w, int64_t N,
                                                         int64_t K, uint8_t* __restrict__ codes,
                                                         float* __restrict__ scales) {
-  griddep_wait();
-  griddep_launch_dependents();
+  griddep_wait();  // no early trigger: a linear call may read these outputs at once
   __shared__ float red[8];
   __shared__ int red_bad[8];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
