@@ -162,7 +162,7 @@ sq_status sq_check(sq_stream_t stream, uint32_t* device_bits) {
   if ((e = take_accept_status(&bits)) != cudaSuccess) return cuda_fail(e, "sq_check: accept status");
   if ((e = take_gemv_status_int4(&bits)) != cudaSuccess ||
       (e = take_gemv_status_fp8(&bits)) != cudaSuccess ||
-      (e = take_gemv_status_fp16(&bits)) != cudaSuccess)
+      (e = take_gemv_status_fp16(&bits)) != cudaSuccess || (e = take_tc_status(&bits)) != cudaSuccess)
     return cuda_fail(e, "sq_check: linear status");
   if (device_bits) *device_bits = bits;
   if (bits) return fail(SQ_ERR_DEVICE, "sq_check: device status bits 0x%x", bits);
@@ -250,7 +250,15 @@ sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void*
   a.row_bytes = row_bytes_of(wkind, K);
   a.pieces = (int)(K / weights_per_piece(wkind));
   a.ppad = (a.pieces + 31) / 32 * 32;
-  cudaError_t e = launch_gemv(wkind, a, (cudaStream_t)stream);
+  cudaError_t e;
+  if (wkind == SQ_W_FP16 && M >= 16 && tc_supported(M, K, epi)) {
+    // a real dense tile: tcgen05 tensor cores, weights on the MMA's M side
+    e = launch_tc_fp16(a.x, reinterpret_cast<const __half*>(w), a.bias, a.residual, a.y, M, N, K, epi,
+                       (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "sq_linear: tensor-core launch");
+    return SQ_OK;
+  }
+  e = launch_gemv(wkind, a, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "sq_linear: launch");
   return SQ_OK;
 }
