@@ -117,13 +117,27 @@ cudaError_t launch_gemv(int wk, const GemvArgs& a0, cudaStream_t st) {
     a.residual = a0.residual ? a0.residual + (int64_t)m0 * a0.N : nullptr;
     const bool silu = a.epi == SQ_EPI_SILU_GATE;
     const int r = (mr <= 5 && a.N >= 8192) ? 2 : 1;
-    const int64_t ntiles = (a.N + r - 1) / r;
+    // lanes per row: the largest of 32/16/8 that divides the row's 16-byte
+    // pieces (no idle lanes), unless that leaves too few tiles to spread
+    // over the GPU's warps; MR >= 8 is compiled for 32 only
+    int lpr = 32;
+    if (mr <= 5) {
+      for (int cand : {32, 16, 8}) {
+        if (a.pieces % cand) continue;
+        const int64_t per_tile = (int64_t)(32 / cand) * r;
+        const int64_t tiles = (a.N + per_tile - 1) / per_tile;
+        if (cand == 32 || tiles >= (int64_t)device_sm_count() * 4) lpr = cand;
+        break;
+      }
+    }
+    const int64_t rows_per_tile = (int64_t)(32 / lpr) * r;
+    const int64_t ntiles = (a.N + rows_per_tile - 1) / rows_per_tile;
     const int64_t blocks = (ntiles + 7) / 8;
     const size_t smem = gemv_smem_bytes(wk, mr, a.K);
     cudaError_t e;
-    if (wk == SQ_W_INT4) e = launch_gemv_int4(a, mr, r, silu, blocks, smem, st);
-    else if (wk == SQ_W_FP8) e = launch_gemv_fp8(a, mr, r, silu, blocks, smem, st);
-    else e = launch_gemv_fp16(a, mr, r, silu, blocks, smem, st);
+    if (wk == SQ_W_INT4) e = launch_gemv_int4(a, mr, r, silu, lpr, blocks, smem, st);
+    else if (wk == SQ_W_FP8) e = launch_gemv_fp8(a, mr, r, silu, lpr, blocks, smem, st);
+    else e = launch_gemv_fp16(a, mr, r, silu, lpr, blocks, smem, st);
     if (e != cudaSuccess) return e;
     m0 += m_here;
   }

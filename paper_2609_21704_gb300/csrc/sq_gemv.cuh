@@ -99,36 +99,44 @@ struct Unroll {
 };
 
 // MR: activation rows compiled for (M <= MR, missing rows read zeros);
-// R: output rows per warp; SILU: fused gate/up epilogue.
-template <int WK, int MR, int R, bool SILU>
+// R: output rows per lane group; SILU: fused gate/up epilogue;
+// LPR: lanes per row.  A warp holds 32 / LPR lane groups, each sweeping its
+// own R rows with LPR lanes; LPR is chosen so that a row's 16-byte pieces
+// divide evenly among the lanes (no idle lanes), and the groups of a warp
+// read the same x slots (shared-memory broadcast).
+template <int WK, int MR, int R, bool SILU, int LPR>
 __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
   using T = WTraits<WK>;
   constexpr int SUB = T::kSub;
-  constexpr int WR = SILU ? 2 * R : R;  // weight rows per warp tile
+  constexpr int WR = SILU ? 2 * R : R;  // weight rows per lane group
   constexpr int U = Unroll<WR>::value;
+  constexpr int GPW = 32 / LPR;         // lane groups per warp
+  constexpr int RPT = GPW * R;          // output rows per warp tile
   extern __shared__ uint4 xs[];
 
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t ntiles = (a.N + R - 1) / R;
+  const int lg = lane / LPR, ll = lane % LPR;
+  const int64_t ntiles = (a.N + RPT - 1) / RPT;
   // this CTA's slice of tiles [t_begin, t_end); warp w takes t_begin + w + 8 i
   const int64_t t_begin = ((int64_t)blockIdx.x * ntiles) / gridDim.x;
   const int64_t t_end = ((int64_t)(blockIdx.x + 1) * ntiles) / gridDim.x;
   const int64_t gwarp = t_begin + warp;
   const int64_t nwarps = kGemvWarps;
-  const int steps = a.ppad / 32;
+  const int steps = (a.pieces + LPR - 1) / LPR;  // pieces of a row per lane
   const int64_t G = a.K / 128;
 
+  auto out_row = [&](int64_t tile, int r) -> int64_t { return tile * RPT + lg * R + (r % R); };
   auto wrow_index = [&](int64_t tile, int r) -> int64_t {
-    if (!SILU) return tile * R + r;
-    return r < R ? tile * R + r : a.N + tile * R + (r - R);
+    return (SILU && r >= R ? a.N : 0) + out_row(tile, r);
   };
   auto row_valid = [&](int64_t tile, int r) -> bool {
-    return tile < t_end && tile * R + (SILU ? (r % R) : r) < a.N;
+    return tile < t_end && out_row(tile, r) < a.N;
   };
-  // L2 bulk prefetch of one tile's rows (lane r < WR takes row r).
+  // L2 bulk prefetch of one tile's rows (lane ll < WR of each group takes
+  // row ll of its group).
   auto prefetch_tile = [&](int64_t tile) {
-    if (lane < WR && row_valid(tile, lane)) {
-      const uint8_t* row = a.w + wrow_index(tile, lane) * a.row_bytes;
+    if (ll < WR && row_valid(tile, ll)) {
+      const uint8_t* row = a.w + wrow_index(tile, ll) * a.row_bytes;
       for (int64_t off = 0; off < a.row_bytes; off += 32768) {
         const int64_t nb = a.row_bytes - off < 32768 ? a.row_bytes - off : 32768;
         prefetch_l2_bulk(row + off, (uint32_t)nb);
@@ -147,7 +155,7 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
       const uint8_t* row = a.w + wi * a.row_bytes;
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        const int p = (jb + u) * 32 + lane;
+        const int p = (jb + u) * LPR + ll;
         const bool in = ok && p < a.pieces;
         wv[u][r] = in ? ld_stream16(row + (int64_t)p * 16) : make_uint4(0u, 0u, 0u, 0u);
         if constexpr (WK == WK_INT4)
@@ -194,7 +202,9 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         const int j = jb + u;
-        if (j * 32 >= a.pieces) break;  // warp-uniform
+        if (j * LPR >= a.pieces) break;  // warp-uniform
+        const int p = j * LPR + ll;      // this lane's piece of the row
+        const int xsl = ((p >> 5) * SUB) * 32 + (p & 31);  // x slot of sub-chunk 0
         if constexpr (WK == WK_INT4) {
           float part[WR][MR];
 #pragma unroll
@@ -212,7 +222,7 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
             }
 #pragma unroll
             for (int m = 0; m < MR; ++m) {
-              const uint4 xq = xs[m * chunks_per_m + (j * SUB + i) * 32 + lane];
+              const uint4 xq = xs[m * chunks_per_m + xsl + i * 32];
 #pragma unroll
               for (int r = 0; r < WR; ++r) part[r][m] = dot8_int4order(c[r], xq, part[r][m]);
             }
@@ -237,7 +247,7 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
             }
 #pragma unroll
             for (int m = 0; m < MR; ++m) {
-              const uint4 xq = xs[m * chunks_per_m + (j * SUB + i) * 32 + lane];
+              const uint4 xq = xs[m * chunks_per_m + xsl + i * 32];
 #pragma unroll
               for (int r = 0; r < WR; ++r)
                 acc[r][m] = dot8_natural(h[r][0], h[r][1], h[r][2], h[r][3], xq, acc[r][m]);
@@ -246,7 +256,7 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
         } else {
 #pragma unroll
           for (int m = 0; m < MR; ++m) {
-            const uint4 xq = xs[m * chunks_per_m + j * 32 + lane];
+            const uint4 xq = xs[m * chunks_per_m + xsl];
 #pragma unroll
             for (int r = 0; r < WR; ++r) {
               const uint4 w = wv[u][r];
@@ -263,16 +273,19 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
 #pragma unroll
     for (int r = 0; r < WR; ++r)
 #pragma unroll
-      for (int m = 0; m < MR; ++m) acc[r][m] = warp_sum(acc[r][m]);
+      for (int m = 0; m < MR; ++m) {
+#pragma unroll
+        for (int o = LPR / 2; o > 0; o >>= 1) acc[r][m] += __shfl_xor_sync(0xffffffffu, acc[r][m], o);
+      }
 
-    // ---- epilogue: lane (r * MR + m) % 32 writes output (r, m)
+    // ---- epilogue: lane (r * MR + m) % LPR of each group writes output (r, m)
 #pragma unroll
     for (int r = 0; r < R; ++r) {
-      const int64_t n = tile * R + r;
+      const int64_t n = out_row(tile, r);
       if (n >= a.N) continue;
 #pragma unroll
       for (int m = 0; m < MR; ++m) {
-        if (m >= a.M || lane != ((r * MR + m) & 31)) continue;
+        if (m >= a.M || ll != ((r * MR + m) % LPR)) continue;
         float v = acc[r][m];
         if constexpr (WK == WK_FP8) v *= reinterpret_cast<const float*>(a.scales)[n];
         if (a.bias) v += __half2float(a.bias[n]);
@@ -292,10 +305,10 @@ __global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
 // Instantiation helper used by the per-format translation units.  The grid
 // is persistent: at most as many CTAs as can be resident at once, each warp
 // looping over the tiles of its CTA's slice.
-template <int WK, int MR, int R, bool SILU>
+template <int WK, int MR, int R, bool SILU, int LPR>
 cudaError_t launch_gemv_inst(const GemvArgs& a, int64_t blocks_needed, size_t smem,
                              cudaStream_t st) {
-  auto k = gemv_kernel<WK, MR, R, SILU>;
+  auto k = gemv_kernel<WK, MR, R, SILU, LPR>;
   struct Cached {
     int smem_set = 0;
     size_t occ_smem[8] = {0};
@@ -331,13 +344,13 @@ cudaError_t launch_gemv_inst(const GemvArgs& a, int64_t blocks_needed, size_t sm
   return launch_pdl(k, dim3(grid > 0 ? grid : 1), dim3(kGemvThreads), smem, st, a);
 }
 
-template <int WK>
-cudaError_t launch_gemv_fmt(const GemvArgs& a, int mr, int r, bool silu, int64_t blocks_needed,
+template <int WK, int LPR>
+cudaError_t launch_gemv_lpr(const GemvArgs& a, int mr, int r, bool silu, int64_t blocks_needed,
                             size_t smem, cudaStream_t st) {
-#define SQ_GEMV_CASE(MR_, R_)                                                              \
-  if (mr == MR_ && r == R_)                                                                \
-    return silu ? launch_gemv_inst<WK, MR_, R_, true>(a, blocks_needed, smem, st)          \
-                : launch_gemv_inst<WK, MR_, R_, false>(a, blocks_needed, smem, st);
+#define SQ_GEMV_CASE(MR_, R_)                                                                  \
+  if (mr == MR_ && r == R_)                                                                    \
+    return silu ? launch_gemv_inst<WK, MR_, R_, true, LPR>(a, blocks_needed, smem, st)         \
+                : launch_gemv_inst<WK, MR_, R_, false, LPR>(a, blocks_needed, smem, st);
   SQ_GEMV_CASE(1, 1)
   SQ_GEMV_CASE(1, 2)
   SQ_GEMV_CASE(2, 1)
@@ -346,10 +359,24 @@ cudaError_t launch_gemv_fmt(const GemvArgs& a, int mr, int r, bool silu, int64_t
   SQ_GEMV_CASE(4, 2)
   SQ_GEMV_CASE(5, 1)
   SQ_GEMV_CASE(5, 2)
-  SQ_GEMV_CASE(8, 1)
-  SQ_GEMV_CASE(16, 1)
 #undef SQ_GEMV_CASE
+  if constexpr (LPR == 32) {
+    if (mr == 8 && r == 1)
+      return silu ? launch_gemv_inst<WK, 8, 1, true, 32>(a, blocks_needed, smem, st)
+                  : launch_gemv_inst<WK, 8, 1, false, 32>(a, blocks_needed, smem, st);
+    if (mr == 16 && r == 1)
+      return silu ? launch_gemv_inst<WK, 16, 1, true, 32>(a, blocks_needed, smem, st)
+                  : launch_gemv_inst<WK, 16, 1, false, 32>(a, blocks_needed, smem, st);
+  }
   return cudaErrorInvalidValue;
+}
+
+template <int WK>
+cudaError_t launch_gemv_fmt(const GemvArgs& a, int mr, int r, bool silu, int lpr,
+                            int64_t blocks_needed, size_t smem, cudaStream_t st) {
+  if (lpr == 16) return launch_gemv_lpr<WK, 16>(a, mr, r, silu, blocks_needed, smem, st);
+  if (lpr == 8) return launch_gemv_lpr<WK, 8>(a, mr, r, silu, blocks_needed, smem, st);
+  return launch_gemv_lpr<WK, 32>(a, mr, r, silu, blocks_needed, smem, st);
 }
 
 // Reads and clears this translation unit's status word.

@@ -5,9 +5,9 @@
 
 namespace sq {
 
-cudaError_t launch_gemv_fp8(const GemvArgs& a, int mr, int r, bool silu, int64_t blocks_needed, size_t smem,
+cudaError_t launch_gemv_fp8(const GemvArgs& a, int mr, int r, bool silu, int lpr, int64_t blocks_needed, size_t smem,
                            cudaStream_t st) {
-  return launch_gemv_fmt<WK_FP8>(a, mr, r, silu, blocks_needed, smem, st);
+  return launch_gemv_fmt<WK_FP8>(a, mr, r, silu, lpr, blocks_needed, smem, st);
 }
 
 cudaError_t take_gemv_status_fp8(uint32_t* bits) { return take_gemv_status_tu(bits); }

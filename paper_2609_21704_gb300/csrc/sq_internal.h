@@ -65,11 +65,11 @@ int gemv_pick_mr(int M);
 cudaError_t launch_gemv(int wkind, const GemvArgs& a, cudaStream_t st);
 // blocks_needed: CTAs that would give every warp one tile; the launcher
 // caps it at the number of CTAs that can be resident at once.
-cudaError_t launch_gemv_int4(const GemvArgs& a, int mr, int r, bool silu, int64_t blocks_needed,
+cudaError_t launch_gemv_int4(const GemvArgs& a, int mr, int r, bool silu, int lpr, int64_t blocks_needed,
                              size_t smem, cudaStream_t st);
-cudaError_t launch_gemv_fp8(const GemvArgs& a, int mr, int r, bool silu, int64_t blocks_needed,
+cudaError_t launch_gemv_fp8(const GemvArgs& a, int mr, int r, bool silu, int lpr, int64_t blocks_needed,
                             size_t smem, cudaStream_t st);
-cudaError_t launch_gemv_fp16(const GemvArgs& a, int mr, int r, bool silu, int64_t blocks_needed,
+cudaError_t launch_gemv_fp16(const GemvArgs& a, int mr, int r, bool silu, int lpr, int64_t blocks_needed,
                              size_t smem, cudaStream_t st);
 cudaError_t take_gemv_status_int4(uint32_t* bits);
 cudaError_t take_gemv_status_fp8(uint32_t* bits);
