@@ -95,7 +95,7 @@ __device__ __forceinline__ float dot8_natural(uint32_t w0, uint32_t w1, uint32_t
 // register budget.
 template <int WR>
 struct Unroll {
-  static constexpr int value = WR == 1 ? 8 : WR == 2 ? 4 : 2;
+  static constexpr int value = WR == 1 ? 12 : WR == 2 ? 4 : 2;
 };
 
 // MR: activation rows compiled for (M <= MR, missing rows read zeros);
