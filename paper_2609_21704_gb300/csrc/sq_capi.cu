@@ -265,10 +265,9 @@ sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void*
   a.pieces = (int)(K / weights_per_piece(wkind));
   a.ppad = (a.pieces + 31) / 32 * 32;
   cudaError_t e;
-  if (wkind == SQ_W_FP16 && M >= 16 && tc_supported(M, K, epi)) {
+  if (M >= 16 && tc_supported(M, K, epi)) {
     // a real dense tile: tcgen05 tensor cores, weights on the MMA's M side
-    e = launch_tc_fp16(a.x, reinterpret_cast<const __half*>(w), a.bias, a.residual, a.y, M, N, K, epi,
-                       (cudaStream_t)stream);
+    e = launch_tc(wkind, a.x, w, scales, a.bias, a.residual, a.y, M, N, K, epi, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "sq_linear: tensor-core launch");
     return SQ_OK;
   }

@@ -75,10 +75,11 @@ cudaError_t take_gemv_status_int4(uint32_t* bits);
 cudaError_t take_gemv_status_fp8(uint32_t* bits);
 cudaError_t take_gemv_status_fp16(uint32_t* bits);
 
-// sq_tc.cu: tcgen05 tensor-core path for M >= 16 (fp16 weights)
+// sq_tc.cu: tcgen05 tensor-core path for M >= 16 (fp16, FP8 or INT4 weights)
 bool tc_supported(int M, int64_t K, int epi);
-cudaError_t launch_tc_fp16(const __half* x, const __half* w, const __half* bias, const __half* residual,
-                           __half* y, int M, int64_t N, int64_t K, int epi, cudaStream_t st);
+cudaError_t launch_tc(int wkind, const __half* x, const void* w, const void* scales, const __half* bias,
+                      const __half* residual, __half* y, int M, int64_t N, int64_t K, int epi,
+                      cudaStream_t st);
 cudaError_t take_tc_status(uint32_t* bits);
 
 // sq_accept.cu

@@ -13,6 +13,16 @@
 // and run the epilogue.  With the fused SiLU gate the CTA also loads the up
 // rows' tile and accumulates a second NB-column block of TMEM.
 //
+// FP8 and INT4 weights: TMA brings the code tiles instead, and the four
+// epilogue warps (idle until the accumulator is final) dequantise each stage
+// into the swizzled fp16 A tile (generic stores, fence.proxy.async, then an
+// mbarrier arrive that releases the stage to the MMA thread).  FP8: exact
+// E4M3 -> fp16, the per-row scale applied in the epilogue (exact).  INT4:
+// c * s rounded once to fp16 (c exact, s the fp16 group scale), a relative
+// rounding of at most 2^-11 per weight, far inside the linear layers' 1e-3
+// relative-L2 tolerance (the per-(row, group) scale cannot be factored out
+// of an MMA that accumulates over several groups).
+//
 // Split-K: the S CTAs of a cluster take consecutive K ranges of the same
 // weight tile; each writes its fp32 partial tile to its own shared memory,
 // and after a cluster barrier CTA r sums rows [r*128/S, (r+1)*128/S) over
@@ -121,6 +131,7 @@ __device__ __forceinline__ float ld_dsmem_f32(const float* local, uint32_t rank)
 // ---------------------------------------------------------------- kernel
 
 struct TcArgs {
+  const void* scales;  // FP8: fp32 [rows]; INT4: fp16 [rows, K/128]; FP16: unused
   int M;            // activation rows present
   int NB;           // MMA N: M rounded up to 16
   int64_t N;        // output columns (weight rows, or gate rows with SILU)
@@ -133,16 +144,20 @@ struct TcArgs {
   uint32_t idesc;
   int stage_bytes;  // A (+ A_up) + B, multiple of 1024
   int b_off;        // offset of B inside a stage
+  int c_off;        // offset of the code tiles inside a stage (FP8 / INT4)
+  int c_bytes;      // bytes of one code tile
   int part_stride;  // floats between columns of the partial tile
   const __half* bias;
   const __half* residual;
   __half* y;
 };
 
-template <bool SILU>
+// WK: 0 fp16 weights, 1 INT4 codes, 2 FP8 codes (the GEMV family's numbering).
+template <int WK, bool SILU>
 __global__ void __launch_bounds__(kTcThreads, 1)
     tc_linear_kernel(const __grid_constant__ CUtensorMap tw, const __grid_constant__ CUtensorMap tx,
                      const TcArgs a) {
+  constexpr bool QUANT = WK != 0;
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the swizzle atoms
   const uint32_t raw = smem_u32(smem_raw);
@@ -152,7 +167,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   uint64_t* full = bars;
   uint64_t* empty = bars + a.nstages;
   uint64_t* accf = bars + 2 * a.nstages;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * a.nstages + 1);
+  uint64_t* conv = bars + 2 * a.nstages + 1;  // converted A tiles ready (quantised weights)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 3 * a.nstages + 1);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int S = a.splits;
@@ -166,6 +182,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     for (int s = 0; s < a.nstages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
+      mbar_init(&conv[s], 4);
     }
     mbar_init(accf, 1);
     fence_mbar_init();
@@ -187,15 +204,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // --------------------------------------------------------- producer
-      const uint32_t bytes = (uint32_t)(kTcStageA * (SILU ? 2 : 1) + a.NB * 128);
+      const uint32_t bytes =
+          (uint32_t)((QUANT ? a.c_bytes : kTcStageA) * (SILU ? 2 : 1) + a.NB * 128);
+      // weight tiles land in A (fp16) or in the code area (quantised)
+      const int wdst = QUANT ? a.c_off : 0;
+      const int wdst_up = QUANT ? a.c_off + a.c_bytes : kTcStageA;
+      // TMA x coordinate of a weight tile: k (fp16, FP8 bytes) or k / 2 (INT4 bytes)
+      auto wx = [&](int k0) { return WK == 1 ? k0 / 2 : k0; };
       const int pre = nk < a.nstages ? nk : a.nstages;
       // weights never depend on the previous kernel: start them first
       for (int it = 0; it < pre; ++it) {
         uint8_t* st = stages + (size_t)it * a.stage_bytes;
         const int k0 = (k_begin + it) * kTcBK;
         mbar_arrive_expect_tx(&full[it], bytes);
-        tma_load_2d(st, &tw, k0, (int)(tile * kTcBM), &full[it]);
-        if (SILU) tma_load_2d(st + kTcStageA, &tw, k0, (int)(a.N + tile * kTcBM), &full[it]);
+        tma_load_2d(st + wdst, &tw, wx(k0), (int)(tile * kTcBM), &full[it]);
+        if (SILU) tma_load_2d(st + wdst_up, &tw, wx(k0), (int)(a.N + tile * kTcBM), &full[it]);
       }
       griddep_wait();
       for (int it = 0; it < pre; ++it)
@@ -211,8 +234,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         uint8_t* st = stages + (size_t)s * a.stage_bytes;
         const int k0 = (k_begin + it) * kTcBK;
         mbar_arrive_expect_tx(&full[s], bytes);
-        tma_load_2d(st, &tw, k0, (int)(tile * kTcBM), &full[s]);
-        if (SILU) tma_load_2d(st + kTcStageA, &tw, k0, (int)(a.N + tile * kTcBM), &full[s]);
+        tma_load_2d(st + wdst, &tw, wx(k0), (int)(tile * kTcBM), &full[s]);
+        if (SILU) tma_load_2d(st + wdst_up, &tw, wx(k0), (int)(a.N + tile * kTcBM), &full[s]);
         tma_load_2d(st + a.b_off, &tx, k0, 0, &full[s]);
       }
     }
@@ -222,7 +245,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int it = 0; it < nk; ++it) {
         const int s = it % a.nstages;
         const uint32_t ph = (uint32_t)(it / a.nstages) & 1u;
-        if (!timed_out && !mbar_wait_bounded(&full[s], ph)) {
+        if (!timed_out && !mbar_wait_bounded(QUANT ? &conv[s] : &full[s], ph)) {
           timed_out = true;
           atomicOr(&g_tc_status, SQ_DEV_TIMEOUT);
         }
@@ -243,8 +266,63 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       tc_commit(accf);
     }
   } else {
-    // ----------------------------------------------------------- epilogue
+    // ------------------------------------- converters (quantised), epilogue
     griddep_wait();
+    if constexpr (QUANT) {
+      const int ct = tid - 64;  // 0..127
+      const int64_t G = a.K / 128;
+      const int64_t wrows = SILU ? 2 * a.N : a.N;
+      for (int it = 0; it < nk; ++it) {
+        const int s = it % a.nstages;
+        const uint32_t ph = (uint32_t)(it / a.nstages) & 1u;
+        if (!timed_out && !mbar_wait_bounded(&full[s], ph)) {
+          timed_out = true;
+          if (lane == 0) atomicOr(&g_tc_status, SQ_DEV_TIMEOUT);
+        }
+        uint8_t* st = stages + (size_t)s * a.stage_bytes;
+        const int g = ((k_begin + it) * kTcBK) >> 7;  // INT4 scale group of this stage
+#pragma unroll
+        for (int h = 0; h < (SILU ? 2 : 1); ++h) {
+          const uint8_t* codes = st + a.c_off + h * a.c_bytes;
+          uint8_t* at = st + h * kTcStageA;
+#pragma unroll 2
+          for (int j = 0; j < 8; ++j) {
+            // 4 rows x 8 chunks per warp and pass: conflict-free reads and writes
+            const int job = j * 128 + ct;
+            const int row = job >> 3, c = job & 7;
+            uint4 out;
+            if constexpr (WK == 2) {
+              const uint2 cw = *reinterpret_cast<const uint2*>(codes + row * 64 + c * 8);
+              out.x = e4m3x2_to_f16x2(lo16(cw.x));
+              out.y = e4m3x2_to_f16x2(hi16(cw.x));
+              out.z = e4m3x2_to_f16x2(lo16(cw.y));
+              out.w = e4m3x2_to_f16x2(hi16(cw.y));
+            } else {
+              const uint32_t cw = *reinterpret_cast<const uint32_t*>(codes + row * 32 + c * 4);
+              uint32_t q[4];
+              int4x8_to_f16x2(cw, q);  // (k0,k4),(k1,k5),(k2,k6),(k3,k7)
+              const int64_t wrow = (h ? a.N : 0) + tile * kTcBM + row;
+              const __half sc = wrow < wrows
+                                    ? __ldg(reinterpret_cast<const __half*>(a.scales) + wrow * G + g)
+                                    : __ushort_as_half(0);
+              const __half2 s2 = __half2half2(sc);
+              auto mul = [&](uint32_t v) {
+                const __half2 r = __hmul2(*reinterpret_cast<const __half2*>(&v), s2);
+                return *reinterpret_cast<const uint32_t*>(&r);
+              };
+              out.x = mul(__byte_perm(q[0], q[1], 0x5410));  // (k0, k1)
+              out.y = mul(__byte_perm(q[2], q[3], 0x5410));  // (k2, k3)
+              out.z = mul(__byte_perm(q[0], q[1], 0x7632));  // (k4, k5)
+              out.w = mul(__byte_perm(q[2], q[3], 0x7632));  // (k6, k7)
+            }
+            *reinterpret_cast<uint4*>(at + row * 128 + ((c ^ (row & 7)) << 4)) = out;
+          }
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&conv[s]);
+      }
+    }
     if (!mbar_wait_bounded(accf, 0u)) {
       timed_out = true;
       if (lane == 0) atomicOr(&g_tc_status, SQ_DEV_TIMEOUT);
@@ -265,9 +343,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int m = c0 + j;
             if (m >= a.M) break;
             float v = g[j];
+            if constexpr (WK == 2) v *= reinterpret_cast<const float*>(a.scales)[n];
             if (a.bias) v += __half2float(a.bias[n]);
             if (SILU) {
               float uu = u[j];
+              if constexpr (WK == 2) uu *= reinterpret_cast<const float*>(a.scales)[a.N + n];
               if (a.bias) uu += __half2float(a.bias[a.N + n]);
               v = v / (1.0f + expf(-v)) * uu;
             }
@@ -308,8 +388,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         if (n < a.N) {
           float v = g;
+          if constexpr (WK == 2) v *= reinterpret_cast<const float*>(a.scales)[n];
           if (a.bias) v += __half2float(a.bias[n]);
           if (SILU) {
+            if constexpr (WK == 2) u *= reinterpret_cast<const float*>(a.scales)[a.N + n];
             if (a.bias) u += __half2float(a.bias[a.N + n]);
             v = v / (1.0f + expf(-v)) * u;
           }
@@ -345,26 +427,27 @@ static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
-// fp16 [rows, K] row-major -> 2-D tensor map, box (64 k, box_rows), 128-byte
-// swizzle, zero fill outside the tensor.
-static bool make_map(CUtensorMap* m, const void* base, int64_t rows, int64_t K, int box_rows) {
+// [rows, inner] row-major -> 2-D tensor map with box (box_inner, box_rows);
+// zero fill outside the tensor.
+static bool make_map(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int elem_bytes,
+                     int64_t rows, int64_t inner, int box_inner, int box_rows,
+                     CUtensorMapSwizzle swz) {
   auto enc = tensor_map_encoder();
   if (!enc) return false;
-  cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)K * 2};
-  cuuint32_t box[2] = {(cuuint32_t)kTcBK, (cuuint32_t)box_rows};
+  cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)inner * (cuuint64_t)elem_bytes};
+  cuuint32_t box[2] = {(cuuint32_t)box_inner, (cuuint32_t)box_rows};
   cuuint32_t estr[2] = {1, 1};
-  return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  return enc(m, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // instruction descriptor, kind::f16: D fp32, A and B fp16, both K-major,
 // N = nb, M = 128
 static uint32_t make_idesc(int nb) {
   uint32_t d = 0;
-  d |= 1u << 4;                  // D format fp32
-  d |= (uint32_t)(nb >> 3) << 17;  // N / 8
+  d |= 1u << 4;                       // D format fp32
+  d |= (uint32_t)(nb >> 3) << 17;     // N / 8
   d |= (uint32_t)(kTcBM >> 4) << 24;  // M / 16
   return d;
 }
@@ -374,60 +457,21 @@ bool tc_supported(int M, int64_t K, int epi) {
   return M >= 16 && M <= 256 && K % 8 == 0 && tensor_map_encoder() != nullptr;
 }
 
-cudaError_t launch_tc_fp16(const __half* x, const __half* w, const __half* bias, const __half* residual,
-                           __half* y, int M, int64_t N, int64_t K, int epi, cudaStream_t st) {
-  const bool silu = epi == SQ_EPI_SILU_GATE;
-  const int nb = (M + 15) / 16 * 16;
-  const int64_t wrows = silu ? 2 * N : N;
-  CUtensorMap tw, tx;
-  if (!make_map(&tw, w, wrows, K, kTcBM) || !make_map(&tx, x, M, K, nb)) return cudaErrorInvalidValue;
-  TcArgs a = {};
-  a.M = M;
-  a.NB = nb;
-  a.N = N;
-  a.K = K;
-  a.epi = epi;
-  a.ksteps = (int)((K + kTcBK - 1) / kTcBK);
-  a.bias = bias;
-  a.residual = residual;
-  a.y = y;
-  a.idesc = make_idesc(nb);
-  const int cols = nb * (silu ? 2 : 1);
-  int tc = 32;
-  while (tc < cols) tc <<= 1;
-  a.tmem_cols = tc;
-  const int a_bytes = kTcStageA * (silu ? 2 : 1);
-  const int b_bytes = (nb * 128 + 1023) / 1024 * 1024;
-  a.b_off = a_bytes;
-  a.stage_bytes = a_bytes + b_bytes;
-  // split K over a cluster until the tiles cover the SMs
-  const int64_t tiles = (N + kTcBM - 1) / kTcBM;
-  const int sms = device_sm_count();
-  int S = 1;
-  while (S < 8 && tiles * S * 2 <= sms && a.ksteps >= 4 * S * 2) S <<= 1;
-  a.splits = S;
-  a.part_stride = kTcBM + 4;
-  const size_t part_bytes = (size_t)cols * a.part_stride * 4;
-  int ns = (int)((200 * 1024) / a.stage_bytes);
-  if (ns > 8) ns = 8;
-  if (ns < 2) ns = 2;
-  while ((size_t)ns * a.stage_bytes < part_bytes) ++ns;
-  a.nstages = ns;
-  const size_t smem = 1024 + (size_t)ns * a.stage_bytes + (2 * ns + 2) * 8 + 16;
-  auto k = silu ? tc_linear_kernel<true> : tc_linear_kernel<false>;
-  static int smem_set[2][64] = {{0}};
+template <int WK, bool SILU>
+static cudaError_t tc_launch_inst(const CUtensorMap& tw, const CUtensorMap& tx, const TcArgs& a,
+                                  int S, int64_t tiles, size_t smem, cudaStream_t st) {
+  auto k = tc_linear_kernel<WK, SILU>;
+  static int smem_set[64] = {0};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if ((int)smem > smem_set[silu][dev]) {
+  if ((int)smem > smem_set[dev]) {
     e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    if (S > 1) {
-      e = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-      if (e != cudaSuccess) return e;
-    }
-    smem_set[silu][dev] = (int)smem;
+    e = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+    smem_set[dev] = (int)smem;
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)S, (unsigned)tiles, 1);
@@ -450,6 +494,78 @@ cudaError_t launch_tc_fp16(const __half* x, const __half* w, const __half* bias,
   cfg.attrs = attr;
   cfg.numAttrs = na;
   return cudaLaunchKernelEx(&cfg, k, tw, tx, a);
+}
+
+cudaError_t launch_tc(int wk, const __half* x, const void* w, const void* scales, const __half* bias,
+                      const __half* residual, __half* y, int M, int64_t N, int64_t K, int epi,
+                      cudaStream_t st) {
+  const bool silu = epi == SQ_EPI_SILU_GATE;
+  const int nb = (M + 15) / 16 * 16;
+  const int64_t wrows = silu ? 2 * N : N;
+  CUtensorMap tw, tx;
+  bool ok;
+  int c_bytes = 0;
+  if (wk == SQ_W_FP16) {
+    ok = make_map(&tw, w, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, wrows, K, kTcBK, kTcBM,
+                  CU_TENSOR_MAP_SWIZZLE_128B);
+  } else if (wk == SQ_W_FP8) {
+    c_bytes = kTcBM * kTcBK;  // 64 codes per row
+    ok = make_map(&tw, w, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, wrows, K, kTcBK, kTcBM,
+                  CU_TENSOR_MAP_SWIZZLE_NONE);
+  } else {
+    c_bytes = kTcBM * kTcBK / 2;  // 64 nibbles = 32 bytes per row
+    ok = make_map(&tw, w, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, wrows, K / 2, kTcBK / 2, kTcBM,
+                  CU_TENSOR_MAP_SWIZZLE_NONE);
+  }
+  ok = ok && make_map(&tx, x, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, M, K, kTcBK, nb,
+                      CU_TENSOR_MAP_SWIZZLE_128B);
+  if (!ok) return cudaErrorInvalidValue;
+  TcArgs a = {};
+  a.scales = scales;
+  a.M = M;
+  a.NB = nb;
+  a.N = N;
+  a.K = K;
+  a.epi = epi;
+  a.ksteps = (int)((K + kTcBK - 1) / kTcBK);
+  a.bias = bias;
+  a.residual = residual;
+  a.y = y;
+  a.idesc = make_idesc(nb);
+  const int S2 = silu ? 2 : 1;
+  const int cols = nb * S2;
+  int tc = 32;
+  while (tc < cols) tc <<= 1;
+  a.tmem_cols = tc;
+  const int a_bytes = kTcStageA * S2;
+  const int b_bytes = (nb * 128 + 1023) / 1024 * 1024;
+  a.b_off = a_bytes;
+  a.c_off = a_bytes + b_bytes;
+  a.c_bytes = c_bytes;
+  a.stage_bytes = a.c_off + (c_bytes * S2 + 1023) / 1024 * 1024;
+  // split K over a cluster until the tiles cover the SMs
+  const int64_t tiles = (N + kTcBM - 1) / kTcBM;
+  const int sms = device_sm_count();
+  int S = 1;
+  while (S < 8 && tiles * S * 2 <= sms && a.ksteps >= 4 * S * 2) S <<= 1;
+  a.splits = S;
+  a.part_stride = kTcBM + 4;
+  const size_t part_bytes = (size_t)cols * a.part_stride * 4;
+  int ns = (int)((200 * 1024) / a.stage_bytes);
+  if (ns > 8) ns = 8;
+  if (ns < 2) ns = 2;
+  while ((size_t)ns * a.stage_bytes < part_bytes) ++ns;
+  a.nstages = ns;
+  const size_t smem = 1024 + (size_t)ns * a.stage_bytes + (3 * ns + 2) * 8 + 16;
+  if (smem > 227 * 1024) return cudaErrorInvalidValue;
+#define SQ_TC_CASE(WK_)                                                                \
+  if (wk == WK_) return silu ? tc_launch_inst<WK_, true>(tw, tx, a, S, tiles, smem, st)  \
+                             : tc_launch_inst<WK_, false>(tw, tx, a, S, tiles, smem, st);
+  SQ_TC_CASE(SQ_W_FP16)
+  SQ_TC_CASE(SQ_W_INT4)
+  SQ_TC_CASE(SQ_W_FP8)
+#undef SQ_TC_CASE
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t take_tc_status(uint32_t* bits) {

@@ -69,3 +69,58 @@ def test_tc_full_size_down_proj_7b_sampled(M):
     w_rows = bits16(wt[torch.from_numpy(cols).to(dev())]).view(np.float16).astype(np.float64)
     x64 = bits16(xt).view(np.float16).astype(np.float64)
     assert_close(dev_to_f64(y)[:, cols], oracle.linear(x64, w_rows), f"7B down M={M}")
+
+
+def _quant_variant(kind, w):
+    N, K = w.shape
+    if kind == "int4":
+        c, s = oracle.quantize_int4(w.view(np.uint16))
+        return torch.from_numpy(c).to(dev()), f16_to_dev(s.view(np.float16)), oracle.dequant_int4(c, s, K)
+    c, s = oracle.quantize_fp8(w.view(np.uint16))
+    return torch.from_numpy(c).to(dev()), torch.from_numpy(s).to(dev()), oracle.dequant_fp8(c, s)
+
+
+WKQ = {"int4": sq.SQ_W_INT4, "fp8": sq.SQ_W_FP8}
+
+
+@pytest.mark.parametrize("kind", ["int4", "fp8"])
+@pytest.mark.parametrize("M", [16, 33, 48, 144])
+@pytest.mark.parametrize("N,K", [(200, 1024), (1536, 1536), (384, 8960)])
+def test_tc_quantised_weights_match_oracle(kind, M, N, K):
+    w = synth.weights_fp16(N * 7 + K + M, N, K)
+    x = synth.activations_fp16(M * 5 + K, M, K)
+    wd, sd, w64 = _quant_variant(kind, w)
+    y = torch.empty(M, N, dtype=torch.float16, device=dev())
+    sq.sq_linear_ex(WKQ[kind], f16_to_dev(x), wd, sd, None, None, sq.SQ_EPI_NONE, y)
+    assert sq.sq_check() == 0
+    assert_close(dev_to_f64(y), oracle.linear(x.astype(np.float64), w64), f"{kind} M={M} N={N} K={K}")
+
+
+@pytest.mark.parametrize("kind", ["int4", "fp8"])
+def test_tc_quantised_silu_bias(kind):
+    I, K, M = 256, 1536, 48
+    w = synth.weights_fp16(51, 2 * I, K)
+    x = synth.activations_fp16(52, M, K)
+    b = synth.fp16_normal(53, (2 * I,), 0.5)
+    wd, sd, w64 = _quant_variant(kind, w)
+    y = torch.empty(M, I, dtype=torch.float16, device=dev())
+    sq.sq_linear_ex(WKQ[kind], f16_to_dev(x), wd, sd, f16_to_dev(b), None, sq.SQ_EPI_SILU_GATE, y)
+    full = oracle.linear(x.astype(np.float64), w64, b.astype(np.float64))
+    assert_close(dev_to_f64(y), oracle.silu_gate(full[:, :I], full[:, I:]), kind)
+
+
+def test_tc_fp8_full_size_qkv_7b_sampled():
+    _, N, K = QWEN25_7B.projections()[0]
+    M = 48
+    wt = synth.weights_fp16_device(61, N, K, dev())
+    codes = torch.empty(N, K, dtype=torch.uint8, device=dev())
+    scales = torch.empty(N, dtype=torch.float32, device=dev())
+    sq.sq_quantize(wt, sq.SQ_FP8_E4M3_ROW, codes, scales)
+    xt = synth.activations_fp16_device(62, M, K, dev())
+    y = torch.empty(M, N, dtype=torch.float16, device=dev())
+    sq.sq_linear_fp8(xt, codes, scales, None, y)
+    cols = np.unique(np.concatenate([[0, N - 1], np.random.default_rng(7).integers(0, N, 62)]))
+    w_rows = bits16(wt[torch.from_numpy(cols).to(dev())]).view(np.float16)
+    c, s = oracle.quantize_fp8(w_rows.view(np.uint16))
+    x64 = bits16(xt).view(np.float16).astype(np.float64)
+    assert_close(dev_to_f64(y)[:, cols], oracle.linear(x64, oracle.dequant_fp8(c, s)), "fp8 7B qkv M=48")
