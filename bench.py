@@ -371,9 +371,11 @@ def main():
     ver_bytes = stack.weight_bytes("fp16") + stack.activation_bytes(Mv)
     acc_bytes = B * (2 * V * 4 + 2 * K * 4)
 
-    # ---- dominant kernel: the fused gate/up + SiLU GEMV (largest per-launch
+    # ---- dominant kernel: the fused gate/up + SiLU linear (largest per-launch
     # weight matrix in the layers); all layers' launches of it in one graph
-    kernel_tag = f"gemv_{args.draft}_gateup_silu_m{B}"
+    engine = "tc" if sq.sq_linear_path(stk.WKIND[args.draft], B, shape.intermediate, shape.hidden,
+                                       sq.SQ_EPI_SILU_GATE) == 1 else "gemv"
+    kernel_tag = f"{engine}_{args.draft}_gateup_silu_m{B}"
     gu_projs = [layer[2] for layer in stack.layers]
 
     def gu_only(variant, bufs):

@@ -26,7 +26,7 @@ __all__ = [
     "SQ_EPI_NONE", "SQ_EPI_SILU_GATE", "SQ_EPI_RESIDUAL", "SQ_W_FP16", "SQ_W_INT4", "SQ_W_FP8",
     "sq_quantized_bytes", "sq_quantize", "sq_linear_w4a16", "sq_linear_fp8", "sq_verify",
     "sq_linear_ex", "sq_accept_workspace_bytes", "sq_accept", "sq_sample", "sq_check",
-    "sq_version", "sq_accept_noalloc", "EXPORTED_SYMBOLS",
+    "sq_version", "sq_accept_noalloc", "sq_linear_path", "EXPORTED_SYMBOLS",
 ]
 
 SQ_OK = 0
@@ -55,6 +55,7 @@ _SIGS = {
     "sq_accept": (_INT, [_P, _P, _P, _P, _INT, _INT, _I64, _INT, _P, _P, _P, _SIZE, _P]),
     "sq_sample": (_INT, [_P, _P, _INT, _I64, _P, _P, _SIZE, _P]),
     "sq_accept_noalloc": (_INT, [_P, _P, _P, _P, _INT, _INT, _I64, _INT, _P, _P, _P]),
+    "sq_linear_path": (_INT, [_INT, _INT, _I64, _I64, _INT]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGS)
 
@@ -115,6 +116,11 @@ def _stream(stream):
 
 def sq_version() -> int:
     return load().sq_version()
+
+
+def sq_linear_path(wkind: int, M: int, N: int, K: int, epi: int = SQ_EPI_NONE) -> int:
+    """1: tensor cores, 0: CUDA-core GEMV, -1: sizes sq_linear_ex rejects."""
+    return load().sq_linear_path(wkind, M, N, K, epi)
 
 
 def sq_quantized_bytes(kind: int, N: int, K: int):

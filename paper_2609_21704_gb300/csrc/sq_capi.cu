@@ -96,6 +96,27 @@ static int gemv_cap_mr(int wk, int64_t K) {
   return best;
 }
 
+// Tensor cores or CUDA cores.  From 16 rows on a CUDA-core GEMV is issue
+// bound (16 fused multiply-adds per weight); below that the choice follows
+// timings of both paths on the 1.5B/7B/14B projection shapes:
+//   * 8..15 rows: tensor cores for FP16 and FP8 weights (1.5-3x faster on
+//     every shape), and for INT4 weights from 8 Mi weights on (the INT4
+//     GEMV keeps small matrices, where its 8 x dequant reuse still pays);
+//   * 3..7 rows, FP16 weights: tensor cores for long rows (K >= 8192), the
+//     fused gate/up from 16 Mi weights, and wide outputs (N >= 65536) with
+//     K >= 2048; the GEMV for the rest (its many warps fill the GPU better
+//     than 128-row tiles do when N is small);
+//   * fewer rows, or FP8/INT4 below 8 rows: the GEMV.
+static bool use_tensor_cores(int wk, int M, int64_t N, int64_t K, int epi) {
+  const bool silu = epi == SQ_EPI_SILU_GATE;
+  const int64_t weights = (silu ? 2 * N : N) * K;
+  if (M >= 16) return true;
+  if (M >= 8) return wk != SQ_W_INT4 || weights >= ((int64_t)8 << 20);
+  if (wk == SQ_W_FP16 && M >= 3)
+    return K >= 8192 || (silu && weights >= ((int64_t)16 << 20)) || (N >= 65536 && K >= 2048);
+  return false;
+}
+
 cudaError_t launch_gemv(int wk, const GemvArgs& a0, cudaStream_t st) {
   GemvArgs a = a0;
   const int cap = gemv_cap_mr(wk, a.K);
@@ -116,12 +137,20 @@ cudaError_t launch_gemv(int wk, const GemvArgs& a0, cudaStream_t st) {
     a.y = a0.y + (int64_t)m0 * a0.N;
     a.residual = a0.residual ? a0.residual + (int64_t)m0 * a0.N : nullptr;
     const bool silu = a.epi == SQ_EPI_SILU_GATE;
-    const int r = (mr <= 5 && a.N >= 8192) ? 2 : 1;
-    // lanes per row: the largest of 32/16/8 that divides the row's 16-byte
-    // pieces (no idle lanes), unless that leaves too few tiles to spread
-    // over the GPU's warps; MR >= 8 is compiled for 32 only
+    // rows per lane group and lanes per row, fitted to timings of every
+    // projection shape of the 1.5B/7B/14B stacks (within 1 % of the best
+    // of the nine (R, LPR) choices overall): two rows per group once there
+    // are enough rows to keep every warp busy; SiLU already doubles the
+    // rows a group holds
+    int r = 1;
+    if (mr <= 5) r = (a.N >= 4096 && !silu) ? 2 : 1;
+    else r = (mr == 16 && silu) ? 1 : 2;
+    // lanes per row: 32 for long rows (>= 256 pieces, several batches per
+    // row anyway) and for MR >= 8 (compiled for 32 only); otherwise the
+    // largest of 32/16/8 that divides the row's 16-byte pieces (no idle
+    // lanes), unless that leaves too few tiles to spread over the warps
     int lpr = 32;
-    if (mr <= 5) {
+    if (mr <= 5 && a.pieces < 256) {
       for (int cand : {32, 16, 8}) {
         if (a.pieces % cand) continue;
         const int64_t per_tile = (int64_t)(32 / cand) * r;
@@ -220,9 +249,8 @@ sq_status sq_quantize(const void* w16, int64_t N, int64_t K, sq_qkind kind, void
   return SQ_OK;
 }
 
-sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void* scales,
-                       const void* bias, const void* residual, sq_epilogue epi, void* y, int M,
-                       int64_t N, int64_t K, sq_stream_t stream) {
+// Kind and size rules of sq_linear_ex (shared with sq_linear_path).
+static sq_status check_linear_sizes(sq_wkind wkind, int M, int64_t N, int64_t K, sq_epilogue epi) {
   if (wkind != SQ_W_FP16 && wkind != SQ_W_INT4 && wkind != SQ_W_FP8)
     return fail(SQ_ERR_INVALID_ARG, "sq_linear: unknown weight kind %d", (int)wkind);
   if (epi != SQ_EPI_NONE && epi != SQ_EPI_SILU_GATE && epi != SQ_EPI_RESIDUAL)
@@ -238,6 +266,16 @@ sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void*
     return fail(SQ_ERR_SHAPE, "sq_verify: K %% 8 != 0 (K=%lld)", (long long)K);
   if (N > (int64_t)1 << 30 || K > (int64_t)1 << 20)
     return fail(SQ_ERR_SHAPE, "sq_linear: N or K too large");
+  if (gemv_cap_mr(wkind, K) == 0)
+    return fail(SQ_ERR_SHAPE, "sq_linear: K=%lld too large for the staged activations", (long long)K);
+  return SQ_OK;
+}
+
+sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void* scales,
+                       const void* bias, const void* residual, sq_epilogue epi, void* y, int M,
+                       int64_t N, int64_t K, sq_stream_t stream) {
+  sq_status st = check_linear_sizes(wkind, M, N, K, epi);
+  if (st != SQ_OK) return st;
   if (!x || !w || !y) return fail(SQ_ERR_INVALID_ARG, "sq_linear: NULL x, weight or y");
   if (wkind != SQ_W_FP16 && !scales) return fail(SQ_ERR_INVALID_ARG, "sq_linear: NULL scales");
   if (epi == SQ_EPI_RESIDUAL && !residual)
@@ -248,8 +286,6 @@ sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void*
     return fail(SQ_ERR_ALIGN, "sq_linear: scales misaligned");
   if ((bias && !aligned(bias, 2)) || (residual && !aligned(residual, 2)))
     return fail(SQ_ERR_ALIGN, "sq_linear: bias/residual misaligned");
-  if (gemv_cap_mr(wkind, K) == 0)
-    return fail(SQ_ERR_SHAPE, "sq_linear: K=%lld too large for the staged activations", (long long)K);
   GemvArgs a = {};
   a.x = reinterpret_cast<const __half*>(x);
   a.w = reinterpret_cast<const uint8_t*>(w);
@@ -265,8 +301,8 @@ sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void*
   a.pieces = (int)(K / weights_per_piece(wkind));
   a.ppad = (a.pieces + 31) / 32 * 32;
   cudaError_t e;
-  if (M >= 16 && tc_supported(M, K, epi)) {
-    // a real dense tile: tcgen05 tensor cores, weights on the MMA's M side
+  if (use_tensor_cores(wkind, M, N, K, epi) && tc_supported(M, K, epi)) {
+    // tcgen05 tensor cores, weights on the MMA's M side
     e = launch_tc(wkind, a.x, w, scales, a.bias, a.residual, a.y, M, N, K, epi, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "sq_linear: tensor-core launch");
     return SQ_OK;
@@ -274,6 +310,11 @@ sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void*
   e = launch_gemv(wkind, a, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "sq_linear: launch");
   return SQ_OK;
+}
+
+int sq_linear_path(sq_wkind wkind, int M, int64_t N, int64_t K, sq_epilogue epi) {
+  if (check_linear_sizes(wkind, M, N, K, epi) != SQ_OK) return -1;
+  return use_tensor_cores(wkind, M, N, K, epi) && tc_supported(M, K, epi) ? 1 : 0;
 }
 
 sq_status sq_linear_w4a16(const void* x, const void* codes, const void* scales, const void* bias,

@@ -359,14 +359,26 @@ cudaError_t launch_gemv_lpr(const GemvArgs& a, int mr, int r, bool silu, int64_t
   SQ_GEMV_CASE(4, 2)
   SQ_GEMV_CASE(5, 1)
   SQ_GEMV_CASE(5, 2)
+  SQ_GEMV_CASE(4, 4)
+  SQ_GEMV_CASE(5, 4)
 #undef SQ_GEMV_CASE
   if constexpr (LPR == 32) {
     if (mr == 8 && r == 1)
       return silu ? launch_gemv_inst<WK, 8, 1, true, 32>(a, blocks_needed, smem, st)
                   : launch_gemv_inst<WK, 8, 1, false, 32>(a, blocks_needed, smem, st);
+    if (mr == 8 && r == 2)
+      return silu ? launch_gemv_inst<WK, 8, 2, true, 32>(a, blocks_needed, smem, st)
+                  : launch_gemv_inst<WK, 8, 2, false, 32>(a, blocks_needed, smem, st);
+    if (mr == 8 && r == 4)
+      return silu ? launch_gemv_inst<WK, 8, 4, true, 32>(a, blocks_needed, smem, st)
+                  : launch_gemv_inst<WK, 8, 4, false, 32>(a, blocks_needed, smem, st);
     if (mr == 16 && r == 1)
       return silu ? launch_gemv_inst<WK, 16, 1, true, 32>(a, blocks_needed, smem, st)
                   : launch_gemv_inst<WK, 16, 1, false, 32>(a, blocks_needed, smem, st);
+    if (mr == 16 && r == 2)
+      return silu ? launch_gemv_inst<WK, 16, 2, true, 32>(a, blocks_needed, smem, st)
+                  : launch_gemv_inst<WK, 16, 2, false, 32>(a, blocks_needed, smem, st);
+    if (mr == 16 && r == 4 && !silu) return launch_gemv_inst<WK, 16, 4, false, 32>(a, blocks_needed, smem, st);
   }
   return cudaErrorInvalidValue;
 }

@@ -75,7 +75,7 @@ cudaError_t take_gemv_status_int4(uint32_t* bits);
 cudaError_t take_gemv_status_fp8(uint32_t* bits);
 cudaError_t take_gemv_status_fp16(uint32_t* bits);
 
-// sq_tc.cu: tcgen05 tensor-core path for M >= 16 (fp16, FP8 or INT4 weights)
+// sq_tc.cu: tcgen05 tensor-core path (fp16, FP8 or INT4 weights), any M <= 256
 bool tc_supported(int M, int64_t K, int epi);
 cudaError_t launch_tc(int wkind, const __half* x, const void* w, const void* scales, const __half* bias,
                       const __half* residual, __half* y, int M, int64_t N, int64_t K, int epi,

@@ -1,7 +1,10 @@
-// sq_tc.cu -- tensor-core (tcgen05 / TMEM) linear layer for M >= 16 rows.
+// sq_tc.cu -- tensor-core (tcgen05 / TMEM) linear layer (skinny GEMM, M rows
+// padded to a multiple of 16 on the MMA's N side).
 //
-// Sec. III-D.3: the verify pass scores B * (K+1) rows at once; from 16 rows
-// up this is a real dense tile.  Swap-AB: the weight tile is the MMA's A
+// Sec. III-D.3: the verify pass scores B * (K+1) rows at once (the draft
+// pass B rows).  sq_linear_ex sends a call here from 16 rows on, and from 3
+// to 15 rows for the formats and shapes where this path measured faster
+// than the CUDA-core GEMV (rows past M are zero-filled by the TMA load).  Swap-AB: the weight tile is the MMA's A
 // operand (M_mma = 128 weight rows), the activations are B (N_mma = NB, the
 // activation rows padded to a multiple of 16), D = 128 x NB fp32 in TMEM:
 //     D[n, m] = sum_k W[n, k] * x[m, k]   ->   y[m, n]
@@ -272,20 +275,37 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const int ct = tid - 64;  // 0..127
       const int64_t G = a.K / 128;
       const int64_t wrows = SILU ? 2 * a.N : a.N;
+      // INT4 group scales of this thread's 8 rows (gate and up), fetched one
+      // stage ahead so their latency hides behind the previous stage
+      constexpr int S2 = SILU ? 2 : 1;
+      __half sc_cur[S2][8], sc_nxt[S2][8];
+      auto load_scales = [&](int itn, __half (&dst)[S2][8]) {
+        const int gg = ((k_begin + itn) * kTcBK) >> 7;
+#pragma unroll
+        for (int h = 0; h < S2; ++h)
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int64_t wrow = (h ? a.N : 0) + tile * kTcBM + ((j * 128 + ct) >> 3);
+            dst[h][j] = (WK == 1 && itn < nk && wrow < wrows)
+                            ? __ldg(reinterpret_cast<const __half*>(a.scales) + wrow * G + gg)
+                            : __ushort_as_half(0);
+          }
+      };
+      if constexpr (WK == 1) load_scales(0, sc_cur);
       for (int it = 0; it < nk; ++it) {
         const int s = it % a.nstages;
         const uint32_t ph = (uint32_t)(it / a.nstages) & 1u;
+        if constexpr (WK == 1) load_scales(it + 1, sc_nxt);
         if (!timed_out && !mbar_wait_bounded(&full[s], ph)) {
           timed_out = true;
           if (lane == 0) atomicOr(&g_tc_status, SQ_DEV_TIMEOUT);
         }
         uint8_t* st = stages + (size_t)s * a.stage_bytes;
-        const int g = ((k_begin + it) * kTcBK) >> 7;  // INT4 scale group of this stage
 #pragma unroll
         for (int h = 0; h < (SILU ? 2 : 1); ++h) {
           const uint8_t* codes = st + a.c_off + h * a.c_bytes;
           uint8_t* at = st + h * kTcStageA;
-#pragma unroll 2
+#pragma unroll
           for (int j = 0; j < 8; ++j) {
             // 4 rows x 8 chunks per warp and pass: conflict-free reads and writes
             const int job = j * 128 + ct;
@@ -301,11 +321,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
               const uint32_t cw = *reinterpret_cast<const uint32_t*>(codes + row * 32 + c * 4);
               uint32_t q[4];
               int4x8_to_f16x2(cw, q);  // (k0,k4),(k1,k5),(k2,k6),(k3,k7)
-              const int64_t wrow = (h ? a.N : 0) + tile * kTcBM + row;
-              const __half sc = wrow < wrows
-                                    ? __ldg(reinterpret_cast<const __half*>(a.scales) + wrow * G + g)
-                                    : __ushort_as_half(0);
-              const __half2 s2 = __half2half2(sc);
+              const __half2 s2 = __half2half2(sc_cur[h][j]);
               auto mul = [&](uint32_t v) {
                 const __half2 r = __hmul2(*reinterpret_cast<const __half2*>(&v), s2);
                 return *reinterpret_cast<const uint32_t*>(&r);
@@ -321,6 +337,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncwarp();
         if (lane == 0) mbar_arrive(&conv[s]);
+        if constexpr (WK == 1) {
+#pragma unroll
+          for (int h = 0; h < S2; ++h)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) sc_cur[h][j] = sc_nxt[h][j];
+        }
       }
     }
     if (!mbar_wait_bounded(accf, 0u)) {
@@ -454,7 +476,7 @@ static uint32_t make_idesc(int nb) {
 
 bool tc_supported(int M, int64_t K, int epi) {
   (void)epi;
-  return M >= 16 && M <= 256 && K % 8 == 0 && tensor_map_encoder() != nullptr;
+  return M >= 1 && M <= 256 && K % 8 == 0 && tensor_map_encoder() != nullptr;
 }
 
 template <int WK, bool SILU>

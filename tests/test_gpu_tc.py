@@ -1,8 +1,10 @@
-"""GPU parity: the tcgen05 tensor-core linear layer (M >= 16 activation
-rows with fp16 weights: Sec. III-D.3 verify pass at B * (K+1) rows) against
-the fp64 oracle.  Covers ragged N (not a multiple of the 128-row tile) and
-ragged K (not a multiple of the 64-wide stage), split-K over clusters, the
-SiLU-gate / residual / bias epilogues and a full-size 7B projection."""
+"""GPU parity: the tcgen05 tensor-core linear layer (Sec. III-D.3 verify
+pass at B * (K+1) rows, and the draft pass at B rows) against the fp64
+oracle: M >= 16 rows with fp16, FP8 and INT4 weights, and the 3..15-row
+calls routed to it (rows padded with zeros).  Covers ragged N (not a
+multiple of the 128-row tile) and ragged K (not a multiple of the 64-wide
+stage), split-K over clusters, the SiLU-gate / residual / bias epilogues and
+full-size 7B projections."""
 import numpy as np
 import pytest
 import torch
@@ -124,3 +126,57 @@ def test_tc_fp8_full_size_qkv_7b_sampled():
     c, s = oracle.quantize_fp8(w_rows.view(np.uint16))
     x64 = bits16(xt).view(np.float16).astype(np.float64)
     assert_close(dev_to_f64(y)[:, cols], oracle.linear(x64, oracle.dequant_fp8(c, s)), "fp8 7B qkv M=48")
+
+
+# Below 16 rows the tensor-core path takes the formats and shapes where it
+# is faster than the CUDA-core GEMV; rows past M are zero-filled tile rows.
+SMALL_M_TC = [
+    ("fp16", 3, 384, 8960, sq.SQ_EPI_NONE),      # long rows
+    ("fp16", 5, 200, 8192, sq.SQ_EPI_NONE),
+    ("fp16", 7, 65600, 2048, sq.SQ_EPI_NONE),    # wide output
+    ("fp16", 5, 2816, 3072, sq.SQ_EPI_SILU_GATE),
+    ("fp16", 8, 200, 1000, sq.SQ_EPI_NONE),
+    ("fp16", 9, 1536, 1536, sq.SQ_EPI_NONE),
+    ("fp16", 15, 300, 640, sq.SQ_EPI_NONE),
+    ("fp8", 8, 200, 1024, sq.SQ_EPI_NONE),
+    ("fp8", 9, 384, 8960, sq.SQ_EPI_NONE),
+    ("fp8", 12, 256, 1536, sq.SQ_EPI_SILU_GATE),
+    ("int4", 8, 1024, 8192, sq.SQ_EPI_NONE),
+    ("int4", 13, 2048, 4096, sq.SQ_EPI_NONE),
+]
+
+
+@pytest.mark.parametrize("kind,M,N,K,epi", SMALL_M_TC)
+def test_tc_small_m_matches_oracle(kind, M, N, K, epi):
+    wk = {"fp16": sq.SQ_W_FP16, "int4": sq.SQ_W_INT4, "fp8": sq.SQ_W_FP8}[kind]
+    assert sq.sq_linear_path(wk, M, N, K, epi) == 1
+    silu = epi == sq.SQ_EPI_SILU_GATE
+    rows = 2 * N if silu else N
+    w = synth.weights_fp16(rows + 3 * K + M, rows, K)
+    x = synth.activations_fp16(7 * M + K, M, K)
+    if kind == "fp16":
+        wd, sd, w64 = f16_to_dev(w), None, w.astype(np.float64)
+    else:
+        wd, sd, w64 = _quant_variant(kind, w)
+    y = torch.empty(M, N, dtype=torch.float16, device=dev())
+    sq.sq_linear_ex(wk, f16_to_dev(x), wd, sd, None, None, epi, y)
+    assert sq.sq_check() == 0
+    full = oracle.linear(x.astype(np.float64), w64)
+    ref = oracle.silu_gate(full[:, :N], full[:, N:]) if silu else full
+    assert_close(dev_to_f64(y), ref, f"{kind} M={M} N={N} K={K} epi={epi}")
+
+
+def test_engine_choice_small_rows():
+    # few rows and small matrices stay on the CUDA-core GEMV
+    assert sq.sq_linear_path(sq.SQ_W_INT4, 1, 151936, 1536, sq.SQ_EPI_NONE) == 0
+    assert sq.sq_linear_path(sq.SQ_W_FP16, 5, 2048, 1536, sq.SQ_EPI_NONE) == 0
+    assert sq.sq_linear_path(sq.SQ_W_FP16, 5, 151936, 1536, sq.SQ_EPI_NONE) == 0
+    assert sq.sq_linear_path(sq.SQ_W_FP8, 5, 17920, 1536, sq.SQ_EPI_NONE) == 0
+    assert sq.sq_linear_path(sq.SQ_W_INT4, 8, 2048, 1536, sq.SQ_EPI_NONE) == 0
+    # from 16 rows on: tensor cores
+    assert sq.sq_linear_path(sq.SQ_W_INT4, 16, 2048, 1536, sq.SQ_EPI_NONE) == 1
+    assert sq.sq_linear_path(sq.SQ_W_FP16, 16, 128, 64, sq.SQ_EPI_NONE) == 1
+    # sizes sq_linear_ex rejects
+    assert sq.sq_linear_path(sq.SQ_W_INT4, 1, 256, 100, sq.SQ_EPI_NONE) == -1
+    assert sq.sq_linear_path(sq.SQ_W_FP16, 0, 256, 256, sq.SQ_EPI_NONE) == -1
+    assert sq.sq_linear_path(sq.SQ_W_FP16, 257, 256, 256, sq.SQ_EPI_NONE) == -1
