@@ -367,6 +367,11 @@ def main():
         t_draft = timed(g_draft, reps) / reps
         t_ver = timed(g_ver, reps) / reps
         t_acc = timed(g_acc, reps) / reps
+        # the same passes as separate sq_linear_ex calls
+        g_draft_u = capture(lambda: stk.run_pass_unchained(stack, args.draft, bd, stream))
+        g_ver_u = capture(lambda: stk.run_pass_unchained(stack, "fp16", bv, stream))
+        t_draft_u = timed(g_draft_u, reps) / reps
+        t_ver_u = timed(g_ver_u, reps) / reps
     draft_bytes = stack.weight_bytes(args.draft) + stack.activation_bytes(B)
     ver_bytes = stack.weight_bytes("fp16") + stack.activation_bytes(Mv)
     acc_bytes = B * (2 * V * 4 + 2 * K * 4)
@@ -472,11 +477,17 @@ def main():
             "draft_pass_ms": 1e3 * t_draft, "draft_pass_gbs": draft_bytes / t_draft / 1e9,
             "verify_pass_ms": 1e3 * t_ver, "verify_pass_gbs": ver_bytes / t_ver / 1e9,
             "accept_ms": 1e3 * t_acc, "accept_gbs": acc_bytes / t_acc / 1e9,
+            "draft_pass_unchained_ms": 1e3 * t_draft_u, "verify_pass_unchained_ms": 1e3 * t_ver_u,
             "draft_pass_frac_of_peak": draft_bytes / t_draft / 1e9 / peak_gbs,
             "verify_pass_frac_of_peak": ver_bytes / t_ver / 1e9 / peak_gbs,
             "fp16_gateup_silu_m%d_us" % Mv: 1e6 * t_gu16,
             "fp16_gateup_silu_gbs": gu16_bytes / t_gu16 / 1e9,
             "launches_per_pass": stack.launches_per_pass(),
+            # the same step time with the paper's measured acceptance rates
+            # (Table II), E[tokens per cycle] = (1 - a^(K+1)) / (1 - a)
+            "projected_tokens_per_s_at_paper_alpha": {
+                str(a_p): B * world * (1.0 - a_p ** (K + 1)) / (1.0 - a_p) / (ms_per_step / 1e3)
+                for a_p in (0.579, 0.661)},
         },
         "roofline": {"bound": "hbm", "kernel": kernel_tag, "achieved": achieved, "peak": peak_gbs,
                      "unit": "GB/s", "frac": achieved / peak_gbs, "traffic": traffic,

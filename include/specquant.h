@@ -161,6 +161,29 @@ SQ_API sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, cons
  * this is introspection for tests and tuning. */
 SQ_API int sq_linear_path(sq_wkind wkind, int M, int64_t N, int64_t K, sq_epilogue epi);
 
+/* Sec. III-D.2 / III-D.3: a draft or verify pass runs every projection of
+ * every layer plus lm_head, one after another.  sq_linear_chain runs `count`
+ * linear calls in order on `stream` with exactly the results of calling
+ * sq_linear_ex on each (an op may read what an earlier op wrote): one host
+ * call per pass.  Every op is checked before the first launch; on an error
+ * nothing is launched and sq_last_error names the op.  `ops` is host memory
+ * read during the call only.  Each op follows sq_linear_ex's rules;
+ * `reserved` must be 0. */
+typedef struct sq_linear_op {
+  sq_wkind wkind;        /* weight format */
+  sq_epilogue epi;       /* epilogue */
+  int M;                 /* activation rows */
+  int reserved;          /* must be 0 */
+  int64_t N, K;          /* output columns, inner size */
+  const void* x;         /* fp16 [M, K] */
+  const void* w;         /* codes, or fp16 [N or 2N, K] */
+  const void* scales;    /* NULL for SQ_W_FP16 */
+  const void* bias;      /* or NULL */
+  const void* residual;  /* read only for SQ_EPI_RESIDUAL */
+  void* y;               /* fp16 [M, N] */
+} sq_linear_op;
+SQ_API sq_status sq_linear_chain(const sq_linear_op* ops, int count, sq_stream_t stream);
+
 /* ------------------------------------------------------------------------
  * Sec. III-A.3 token rule and Sec. III-D.4 acceptance / correction, for a
  * batch of B independent sequences with K draft tokens each over a

@@ -26,7 +26,8 @@ __all__ = [
     "SQ_EPI_NONE", "SQ_EPI_SILU_GATE", "SQ_EPI_RESIDUAL", "SQ_W_FP16", "SQ_W_INT4", "SQ_W_FP8",
     "sq_quantized_bytes", "sq_quantize", "sq_linear_w4a16", "sq_linear_fp8", "sq_verify",
     "sq_linear_ex", "sq_accept_workspace_bytes", "sq_accept", "sq_sample", "sq_check",
-    "sq_version", "sq_accept_noalloc", "sq_linear_path", "EXPORTED_SYMBOLS",
+    "sq_version", "sq_accept_noalloc", "sq_linear_path", "sq_linear_chain", "SqLinearOp",
+    "EXPORTED_SYMBOLS",
 ]
 
 SQ_OK = 0
@@ -56,6 +57,7 @@ _SIGS = {
     "sq_sample": (_INT, [_P, _P, _INT, _I64, _P, _P, _SIZE, _P]),
     "sq_accept_noalloc": (_INT, [_P, _P, _P, _P, _INT, _INT, _I64, _INT, _P, _P, _P]),
     "sq_linear_path": (_INT, [_INT, _INT, _I64, _I64, _INT]),
+    "sq_linear_chain": (_INT, [_P, _INT, _P]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGS)
 
@@ -141,6 +143,24 @@ def sq_linear_ex(wkind, x, w, scales, bias, residual, epi, y, stream=None) -> No
     _check("sq_linear_ex", load().sq_linear_ex(wkind, _ptr(x), _ptr(w), _ptr(scales), _ptr(bias),
                                                _ptr(residual), epi, _ptr(y), M, N, K,
                                                _stream(stream)))
+
+
+class SqLinearOp(ctypes.Structure):
+    """Mirror of the C struct sq_linear_op."""
+    _fields_ = [("wkind", ctypes.c_int), ("epi", ctypes.c_int), ("M", ctypes.c_int),
+                ("reserved", ctypes.c_int), ("N", ctypes.c_int64), ("K", ctypes.c_int64),
+                ("x", _P), ("w", _P), ("scales", _P), ("bias", _P), ("residual", _P), ("y", _P)]
+
+
+def sq_linear_chain(ops, stream=None) -> None:
+    """ops: sequence of (wkind, x, w, scales, bias, residual, epi, y) with the
+    same meaning as sq_linear_ex's arguments; run in order (one C call)."""
+    arr = (SqLinearOp * max(1, len(ops)))()
+    for i, (wkind, x, w, scales, bias, residual, epi, y) in enumerate(ops):
+        M, K = x.shape
+        arr[i] = SqLinearOp(wkind, epi, M, 0, y.shape[1], K, _ptr(x), _ptr(w), _ptr(scales),
+                            _ptr(bias), _ptr(residual), _ptr(y))
+    _check("sq_linear_chain", load().sq_linear_chain(ctypes.cast(arr, _P), len(ops), _stream(stream)))
 
 
 def sq_linear_w4a16(x, codes, scales, bias, y, stream=None) -> None:

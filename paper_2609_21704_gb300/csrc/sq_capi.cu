@@ -271,44 +271,88 @@ static sq_status check_linear_sizes(sq_wkind wkind, int M, int64_t N, int64_t K,
   return SQ_OK;
 }
 
-sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void* scales,
-                       const void* bias, const void* residual, sq_epilogue epi, void* y, int M,
-                       int64_t N, int64_t K, sq_stream_t stream) {
-  sq_status st = check_linear_sizes(wkind, M, N, K, epi);
-  if (st != SQ_OK) return st;
-  if (!x || !w || !y) return fail(SQ_ERR_INVALID_ARG, "sq_linear: NULL x, weight or y");
-  if (wkind != SQ_W_FP16 && !scales) return fail(SQ_ERR_INVALID_ARG, "sq_linear: NULL scales");
-  if (epi == SQ_EPI_RESIDUAL && !residual)
+// Pointer and alignment rules of one linear call.
+static sq_status check_linear_ptrs(const sq_linear_op& op) {
+  if (!op.x || !op.w || !op.y) return fail(SQ_ERR_INVALID_ARG, "sq_linear: NULL x, weight or y");
+  if (op.wkind != SQ_W_FP16 && !op.scales) return fail(SQ_ERR_INVALID_ARG, "sq_linear: NULL scales");
+  if (op.epi == SQ_EPI_RESIDUAL && !op.residual)
     return fail(SQ_ERR_INVALID_ARG, "sq_linear: SQ_EPI_RESIDUAL needs a residual");
-  if (!aligned(x, 16) || !aligned(w, 16) || !aligned(y, 2))
+  if (!aligned(op.x, 16) || !aligned(op.w, 16) || !aligned(op.y, 2))
     return fail(SQ_ERR_ALIGN, "sq_linear: x and weights must be 16-byte aligned, y 2-byte aligned");
-  if (scales && !aligned(scales, wkind == SQ_W_FP8 ? 4 : 2))
+  if (op.scales && !aligned(op.scales, op.wkind == SQ_W_FP8 ? 4 : 2))
     return fail(SQ_ERR_ALIGN, "sq_linear: scales misaligned");
-  if ((bias && !aligned(bias, 2)) || (residual && !aligned(residual, 2)))
+  if ((op.bias && !aligned(op.bias, 2)) || (op.residual && !aligned(op.residual, 2)))
     return fail(SQ_ERR_ALIGN, "sq_linear: bias/residual misaligned");
+  return SQ_OK;
+}
+
+static sq_status check_linear(const sq_linear_op& op) {
+  if (op.reserved != 0) return fail(SQ_ERR_INVALID_ARG, "sq_linear_chain: reserved field must be 0");
+  sq_status st = check_linear_sizes(op.wkind, op.M, op.N, op.K, op.epi);
+  if (st != SQ_OK) return st;
+  return check_linear_ptrs(op);
+}
+
+// Launches one checked call.
+static sq_status run_linear(const sq_linear_op& op, cudaStream_t stream) {
   GemvArgs a = {};
-  a.x = reinterpret_cast<const __half*>(x);
-  a.w = reinterpret_cast<const uint8_t*>(w);
-  a.scales = scales;
-  a.bias = reinterpret_cast<const __half*>(bias);
-  a.residual = epi == SQ_EPI_RESIDUAL ? reinterpret_cast<const __half*>(residual) : nullptr;
-  a.y = reinterpret_cast<__half*>(y);
-  a.M = M;
-  a.epi = epi;
-  a.N = N;
-  a.K = K;
-  a.row_bytes = row_bytes_of(wkind, K);
-  a.pieces = (int)(K / weights_per_piece(wkind));
+  a.x = reinterpret_cast<const __half*>(op.x);
+  a.w = reinterpret_cast<const uint8_t*>(op.w);
+  a.scales = op.scales;
+  a.bias = reinterpret_cast<const __half*>(op.bias);
+  a.residual = op.epi == SQ_EPI_RESIDUAL ? reinterpret_cast<const __half*>(op.residual) : nullptr;
+  a.y = reinterpret_cast<__half*>(op.y);
+  a.M = op.M;
+  a.epi = op.epi;
+  a.N = op.N;
+  a.K = op.K;
+  a.row_bytes = row_bytes_of(op.wkind, op.K);
+  a.pieces = (int)(op.K / weights_per_piece(op.wkind));
   a.ppad = (a.pieces + 31) / 32 * 32;
   cudaError_t e;
-  if (use_tensor_cores(wkind, M, N, K, epi) && tc_supported(M, K, epi)) {
+  if (use_tensor_cores(op.wkind, op.M, op.N, op.K, op.epi) && tc_supported(op.M, op.K, op.epi)) {
     // tcgen05 tensor cores, weights on the MMA's M side
-    e = launch_tc(wkind, a.x, w, scales, a.bias, a.residual, a.y, M, N, K, epi, (cudaStream_t)stream);
+    e = launch_tc(op.wkind, a.x, op.w, op.scales, a.bias, a.residual, a.y, op.M, op.N, op.K, op.epi,
+                  stream);
     if (e != cudaSuccess) return cuda_fail(e, "sq_linear: tensor-core launch");
     return SQ_OK;
   }
-  e = launch_gemv(wkind, a, (cudaStream_t)stream);
+  e = launch_gemv(op.wkind, a, stream);
   if (e != cudaSuccess) return cuda_fail(e, "sq_linear: launch");
+  return SQ_OK;
+}
+
+sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void* scales,
+                       const void* bias, const void* residual, sq_epilogue epi, void* y, int M,
+                       int64_t N, int64_t K, sq_stream_t stream) {
+  sq_linear_op op = {};
+  op.wkind = wkind;
+  op.epi = epi;
+  op.M = M;
+  op.N = N;
+  op.K = K;
+  op.x = x;
+  op.w = w;
+  op.scales = scales;
+  op.bias = bias;
+  op.residual = residual;
+  op.y = y;
+  sq_status st = check_linear(op);
+  if (st != SQ_OK) return st;
+  return run_linear(op, (cudaStream_t)stream);
+}
+
+sq_status sq_linear_chain(const sq_linear_op* ops, int count, sq_stream_t stream) {
+  if (count < 0 || (count > 0 && !ops))
+    return fail(SQ_ERR_INVALID_ARG, "sq_linear_chain: need ops and count >= 0");
+  for (int i = 0; i < count; ++i) {
+    sq_status st = check_linear(ops[i]);
+    if (st != SQ_OK) return fail(st, "sq_linear_chain: op %d: %s", i, g_last_error.c_str());
+  }
+  for (int i = 0; i < count; ++i) {
+    sq_status st = run_linear(ops[i], (cudaStream_t)stream);
+    if (st != SQ_OK) return fail(st, "sq_linear_chain: op %d: %s", i, g_last_error.c_str());
+  }
   return SQ_OK;
 }
 

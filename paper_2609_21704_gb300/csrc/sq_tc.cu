@@ -48,6 +48,7 @@ constexpr int kTcBM = 128;      // weight rows per tile (MMA M)
 constexpr int kTcBK = 64;       // k per stage: 64 fp16 = one 128-byte swizzle row
 constexpr int kTcThreads = 192;  // warp 0 TMA, warp 1 MMA + TMEM, warps 2..5 epilogue
 constexpr int kTcStageA = kTcBM * kTcBK * 2;  // 16 KB
+constexpr int kTcMaxSplit = 8;  // CTAs per cluster along K (portable cluster size)
 
 // ---------------------------------------------------------------- PTX
 
@@ -397,11 +398,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     cluster_sync();  // every partial tile is written
     if (warp >= 2) {
       const int et = tid - 64;  // 0..127
-      const int rows = kTcBM / S;
+      const int rows = (kTcBM + S - 1) / S;  // this rank's rows [r0, r0 + nr)
       const int r0 = (int)rank * rows;
+      const int nr = rows < kTcBM - r0 ? rows : kTcBM - r0;
       const float* part = reinterpret_cast<const float*>(stages);
-      for (int idx = et; idx < rows * a.M; idx += 128) {
-        const int m = idx / rows, row = r0 + (idx - m * rows);
+      for (int idx = et; idx < nr * a.M; idx += 128) {
+        const int m = idx / nr, row = r0 + (idx - m * nr);
         const int64_t n = tile * kTcBM + row;
         float g = 0.0f, u = 0.0f;
         for (int qq = 0; qq < S; ++qq) {
@@ -479,9 +481,10 @@ bool tc_supported(int M, int64_t K, int epi) {
   return M >= 1 && M <= 256 && K % 8 == 0 && tensor_map_encoder() != nullptr;
 }
 
+// Raises the kernel's dynamic shared-memory limit to `smem` (once per size
+// and device) and allows cluster sizes above 8.
 template <int WK, bool SILU>
-static cudaError_t tc_launch_inst(const CUtensorMap& tw, const CUtensorMap& tx, const TcArgs& a,
-                                  int S, int64_t tiles, size_t smem, cudaStream_t st) {
+static cudaError_t tc_prepare(size_t smem) {
   auto k = tc_linear_kernel<WK, SILU>;
   static int smem_set[64] = {0};
   int dev = 0;
@@ -495,6 +498,87 @@ static cudaError_t tc_launch_inst(const CUtensorMap& tw, const CUtensorMap& tx, 
     if (e != cudaSuccess) return e;
     smem_set[dev] = (int)smem;
   }
+  return cudaSuccess;
+}
+
+// Clusters of S CTAs (with `smem` bytes each) that can be resident at once,
+// from the occupancy calculator; cached per device, S and size.
+template <int WK, bool SILU>
+static int tc_max_clusters(int S, size_t smem) {
+  struct Entry {
+    size_t smem;
+    int n;
+  };
+  static Entry cache[64][kTcMaxSplit + 1][4] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64 || S < 1 || S > kTcMaxSplit) return 0;
+  for (Entry& en : cache[dev][S])
+    if (en.smem == smem + 1) return en.n;
+  if (tc_prepare<WK, SILU>(smem) != cudaSuccess) return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)S, 1, 1);
+  cfg.blockDim = dim3(kTcThreads);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)S;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, tc_linear_kernel<WK, SILU>, &cfg) != cudaSuccess) {
+    (void)cudaGetLastError();
+    n = 0;
+  }
+  for (Entry& en : cache[dev][S])
+    if (en.smem == 0) {
+      en.smem = smem + 1;
+      en.n = n;
+      break;
+    }
+  return n;
+}
+
+// Split-K factor.  FP16 and FP8 weights (HBM-bound): double S while the
+// split tiles still fill at most half the SMs, so that the next kernel's
+// CTAs find free SMs and start their weight loads early (programmatic
+// dependent launch) -- filling every SM measured slower on the 7B shapes.
+// INT4 weights (bound by the in-CTA dequantisation): the S in
+// 1..kTcMaxSplit that minimises (waves of resident clusters) x (k-steps per
+// CTA + 2 for the split reduction), at least 2 k-steps per CTA; ties keep
+// the smaller S.
+template <int WK, bool SILU>
+static int tc_pick_split(int64_t tiles, int ksteps, size_t smem) {
+  if (WK != 1) {
+    const int sms = device_sm_count();
+    int S = 1;
+    while (S < kTcMaxSplit && tiles * S * 2 <= sms && ksteps >= 4 * S * 2) S <<= 1;
+    return S;
+  }
+  int best_s = 1;
+  int64_t best = INT64_MAX;
+  for (int S = 1; S <= kTcMaxSplit && ksteps >= 2 * S; ++S) {
+    const int nc = tc_max_clusters<WK, SILU>(S, smem);
+    if (nc <= 0) continue;
+    const int64_t waves = (tiles + nc - 1) / nc;
+    const int64_t cost = waves * ((ksteps + S - 1) / S + (S > 1 ? 2 : 0));
+    if (cost < best) {
+      best = cost;
+      best_s = S;
+    }
+  }
+  return best_s;
+}
+
+template <int WK, bool SILU>
+static cudaError_t tc_launch_inst(const CUtensorMap& tw, const CUtensorMap& tx, TcArgs a,
+                                  int64_t tiles, size_t smem, cudaStream_t st) {
+  auto k = tc_linear_kernel<WK, SILU>;
+  cudaError_t e = tc_prepare<WK, SILU>(smem);
+  if (e != cudaSuccess) return e;
+  const int S = tc_pick_split<WK, SILU>(tiles, a.ksteps, smem);
+  a.splits = S;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)S, (unsigned)tiles, 1);
   cfg.blockDim = dim3(kTcThreads);
@@ -565,12 +649,8 @@ cudaError_t launch_tc(int wk, const __half* x, const void* w, const void* scales
   a.c_off = a_bytes + b_bytes;
   a.c_bytes = c_bytes;
   a.stage_bytes = a.c_off + (c_bytes * S2 + 1023) / 1024 * 1024;
-  // split K over a cluster until the tiles cover the SMs
+  // the split of K over a cluster is chosen per kernel instance (occupancy)
   const int64_t tiles = (N + kTcBM - 1) / kTcBM;
-  const int sms = device_sm_count();
-  int S = 1;
-  while (S < 8 && tiles * S * 2 <= sms && a.ksteps >= 4 * S * 2) S <<= 1;
-  a.splits = S;
   a.part_stride = kTcBM + 4;
   const size_t part_bytes = (size_t)cols * a.part_stride * 4;
   int ns = (int)((200 * 1024) / a.stage_bytes);
@@ -581,8 +661,8 @@ cudaError_t launch_tc(int wk, const __half* x, const void* w, const void* scales
   const size_t smem = 1024 + (size_t)ns * a.stage_bytes + (3 * ns + 2) * 8 + 16;
   if (smem > 227 * 1024) return cudaErrorInvalidValue;
 #define SQ_TC_CASE(WK_)                                                                \
-  if (wk == WK_) return silu ? tc_launch_inst<WK_, true>(tw, tx, a, S, tiles, smem, st)  \
-                             : tc_launch_inst<WK_, false>(tw, tx, a, S, tiles, smem, st);
+  if (wk == WK_) return silu ? tc_launch_inst<WK_, true>(tw, tx, a, tiles, smem, st)  \
+                             : tc_launch_inst<WK_, false>(tw, tx, a, tiles, smem, st);
   SQ_TC_CASE(SQ_W_FP16)
   SQ_TC_CASE(SQ_W_INT4)
   SQ_TC_CASE(SQ_W_FP8)

@@ -28,7 +28,8 @@ from dataclasses import dataclass
 import torch
 
 from . import (SQ_EPI_NONE, SQ_EPI_SILU_GATE, SQ_FP8_E4M3_ROW, SQ_INT4_G128, SQ_W_FP8,
-               SQ_W_FP16, SQ_W_INT4, sq_linear_ex, sq_quantize, sq_quantized_bytes, synth)
+               SQ_W_FP16, SQ_W_INT4, sq_linear_chain, sq_linear_ex, sq_quantize,
+               sq_quantized_bytes, synth)
 from .shapes import StackShape
 
 WKIND = {"fp16": SQ_W_FP16, "int4": SQ_W_INT4, "fp8": SQ_W_FP8}
@@ -137,20 +138,29 @@ class PassBuffers:
         self.attn = self.qkv.view(-1)[: M * sh.q_out].view(M, sh.q_out)
 
 
-def run_pass(stack: LinearStack, variant: str, b: PassBuffers, stream=None) -> None:
-    """One draft (variant int4/fp8) or verify (fp16, or fp8) pass: every
-    projection of every layer plus lm_head, in decoder order."""
+def pass_ops(stack: LinearStack, variant: str, b: PassBuffers):
+    """The linear calls of one pass in decoder order, as sq_linear_chain ops."""
     wk = WKIND[variant]
+    ops = []
     for layer in stack.layers:
         qkv, o, gu, down = layer
-        w, s = qkv.weight(variant)
-        sq_linear_ex(wk, b.x, w, s, None, None, SQ_EPI_NONE, b.qkv, stream)
-        w, s = o.weight(variant)
-        sq_linear_ex(wk, b.attn, w, s, None, None, SQ_EPI_NONE, b.o, stream)
-        w, s = gu.weight(variant)
-        sq_linear_ex(wk, b.x, w, s, None, None, SQ_EPI_SILU_GATE, b.h, stream)
-        w, s = down.weight(variant)
-        sq_linear_ex(wk, b.h, w, s, None, None, SQ_EPI_NONE, b.d, stream)
+        ops.append((wk, b.x, *qkv.weight(variant), None, None, SQ_EPI_NONE, b.qkv))
+        ops.append((wk, b.attn, *o.weight(variant), None, None, SQ_EPI_NONE, b.o))
+        ops.append((wk, b.x, *gu.weight(variant), None, None, SQ_EPI_SILU_GATE, b.h))
+        ops.append((wk, b.h, *down.weight(variant), None, None, SQ_EPI_NONE, b.d))
     if stack.lm_head is not None:
-        w, s = stack.lm_head.weight(variant)
-        sq_linear_ex(wk, b.x, w, s, None, None, SQ_EPI_NONE, b.logits, stream)
+        ops.append((wk, b.x, *stack.lm_head.weight(variant), None, None, SQ_EPI_NONE, b.logits))
+    return ops
+
+
+def run_pass(stack: LinearStack, variant: str, b: PassBuffers, stream=None) -> None:
+    """One draft (variant int4/fp8) or verify (fp16, or fp8) pass: every
+    projection of every layer plus lm_head, in decoder order, as one
+    sq_linear_chain call."""
+    sq_linear_chain(pass_ops(stack, variant, b), stream)
+
+
+def run_pass_unchained(stack: LinearStack, variant: str, b: PassBuffers, stream=None) -> None:
+    """The same pass as separate sq_linear_ex calls."""
+    for (wk, x, w, s, bias, res, epi, y) in pass_ops(stack, variant, b):
+        sq_linear_ex(wk, x, w, s, bias, res, epi, y, stream)
