@@ -46,7 +46,15 @@ static __device__ unsigned int g_tc_status;
 
 constexpr int kTcBM = 128;      // weight rows per tile (MMA M)
 constexpr int kTcBK = 64;       // k per stage: 64 fp16 = one 128-byte swizzle row
-constexpr int kTcThreads = 192;  // warp 0 TMA, warp 1 MMA + TMEM, warps 2..5 epilogue
+// Warp roles: warp 0 TMA, warp 1 MMA + TMEM, warps 2..5 epilogue (one TMEM
+// sub-partition each).  Quantised weights add converter warps: warps 2..
+// 2 + warps - 1 dequantise each stage (two per SM sub-partition, so that
+// one's dependent chain hides behind the other's).
+template <int WK>
+struct TcConv {
+  static constexpr int warps = WK == 0 ? 4 : 8;
+  static constexpr int threads = 64 + 32 * warps;
+};
 constexpr int kTcStageA = kTcBM * kTcBK * 2;  // 16 KB
 constexpr int kTcMaxSplit = 8;  // CTAs per cluster along K (portable cluster size)
 
@@ -151,6 +159,9 @@ struct TcArgs {
   int c_off;        // offset of the code tiles inside a stage (FP8 / INT4)
   int c_bytes;      // bytes of one code tile
   int part_stride;  // floats between columns of the partial tile
+  int sc_off;       // INT4: byte offset of the CTA's group-scale block
+  int sc_ng;        // INT4: groups per row held in the block (>= any CTA's need)
+  int max_split;    // largest split-K factor whose partial tile fits in the stages
   const __half* bias;
   const __half* residual;
   __half* y;
@@ -158,7 +169,7 @@ struct TcArgs {
 
 // WK: 0 fp16 weights, 1 INT4 codes, 2 FP8 codes (the GEMV family's numbering).
 template <int WK, bool SILU>
-__global__ void __launch_bounds__(kTcThreads, 1)
+__global__ void __launch_bounds__(TcConv<WK>::threads, 1)
     tc_linear_kernel(const __grid_constant__ CUtensorMap tw, const __grid_constant__ CUtensorMap tx,
                      const TcArgs a) {
   constexpr bool QUANT = WK != 0;
@@ -166,12 +177,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   // 1024-byte alignment for the swizzle atoms
   const uint32_t raw = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+  // a ring of stages [A (gate, up) | B | codes (gate, up; quantised only)]:
+  // TMA brings B and either the fp16 A tiles or the code tiles, which the
+  // converter warps dequantise into the stage's A tiles
   uint8_t* stages = smem;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)a.nstages * a.stage_bytes);
-  uint64_t* full = bars;
-  uint64_t* empty = bars + a.nstages;
-  uint64_t* accf = bars + 2 * a.nstages;
-  uint64_t* conv = bars + 2 * a.nstages + 1;  // converted A tiles ready (quantised weights)
+  uint64_t* full = bars;                       // stage landed (TMA)
+  uint64_t* empty = bars + a.nstages;          // stage free again (MMA commit)
+  uint64_t* accf = bars + 2 * a.nstages;       // accumulator final
+  uint64_t* conv = bars + 2 * a.nstages + 1;   // A tiles converted (quantised)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 3 * a.nstages + 1);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -186,7 +200,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     for (int s = 0; s < a.nstages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
-      mbar_init(&conv[s], 4);
+      mbar_init(&conv[s], TcConv<WK>::warps);
     }
     mbar_init(accf, 1);
     fence_mbar_init();
@@ -210,7 +224,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       // --------------------------------------------------------- producer
       const uint32_t bytes =
           (uint32_t)((QUANT ? a.c_bytes : kTcStageA) * (SILU ? 2 : 1) + a.NB * 128);
-      // weight tiles land in A (fp16) or in the code area (quantised)
+      // weight tiles land in A (fp16) or in the stage's code area (quantised)
       const int wdst = QUANT ? a.c_off : 0;
       const int wdst_up = QUANT ? a.c_off + a.c_bytes : kTcStageA;
       // TMA x coordinate of a weight tile: k (fp16, FP8 bytes) or k / 2 (INT4 bytes)
@@ -271,32 +285,37 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
   } else {
     // ------------------------------------- converters (quantised), epilogue
+    if constexpr (QUANT) {
+      if constexpr (WK == 1) {
+        // INT4: this CTA's group scales (128 rows x the groups its K range
+        // touches, gate and up) into shared memory once, before waiting on
+        // the previous kernel: scales never depend on it, and the per-stage
+        // conversion then never waits on a global load
+        const int ct = tid - 64;
+        const int64_t G = a.K / 128;
+        const int64_t wrows = SILU ? 2 * a.N : a.N;
+        const int g_lo = (k_begin * kTcBK) >> 7;
+        const int ng = nk > 0 ? (((k_end * kTcBK) - 1) >> 7) + 1 - g_lo : 0;
+        __half* sblk = reinterpret_cast<__half*>(smem + a.sc_off);
+        for (int r = ct; r < (SILU ? 2 : 1) * kTcBM; r += 32 * TcConv<WK>::warps) {
+          const int h = r / kTcBM, rr = r - h * kTcBM;
+          const int64_t wrow = (h ? a.N : 0) + tile * kTcBM + rr;
+          const __half* src = reinterpret_cast<const __half*>(a.scales) + wrow * G + g_lo;
+          __half* dst = sblk + (size_t)r * a.sc_ng;
+          for (int gi = 0; gi < ng; ++gi) dst[gi] = wrow < wrows ? __ldg(src + gi) : __ushort_as_half(0);
+        }
+        named_bar_sync(1, 32 * TcConv<WK>::warps);  // the converter warps
+      }
+    }
     griddep_wait();
     if constexpr (QUANT) {
-      const int ct = tid - 64;  // 0..127
-      const int64_t G = a.K / 128;
-      const int64_t wrows = SILU ? 2 * a.N : a.N;
-      // INT4 group scales of this thread's 8 rows (gate and up), fetched one
-      // stage ahead so their latency hides behind the previous stage
-      constexpr int S2 = SILU ? 2 : 1;
-      __half sc_cur[S2][8], sc_nxt[S2][8];
-      auto load_scales = [&](int itn, __half (&dst)[S2][8]) {
-        const int gg = ((k_begin + itn) * kTcBK) >> 7;
-#pragma unroll
-        for (int h = 0; h < S2; ++h)
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const int64_t wrow = (h ? a.N : 0) + tile * kTcBM + ((j * 128 + ct) >> 3);
-            dst[h][j] = (WK == 1 && itn < nk && wrow < wrows)
-                            ? __ldg(reinterpret_cast<const __half*>(a.scales) + wrow * G + gg)
-                            : __ushort_as_half(0);
-          }
-      };
-      if constexpr (WK == 1) load_scales(0, sc_cur);
+      const int ct = tid - 64;  // 0 .. 32 * converter warps - 1
+      const int g_lo = (k_begin * kTcBK) >> 7;
+      const __half* sblk = reinterpret_cast<const __half*>(smem + a.sc_off);
       for (int it = 0; it < nk; ++it) {
         const int s = it % a.nstages;
         const uint32_t ph = (uint32_t)(it / a.nstages) & 1u;
-        if constexpr (WK == 1) load_scales(it + 1, sc_nxt);
+        const int gi = (((k_begin + it) * kTcBK) >> 7) - g_lo;  // this stage's group
         if (!timed_out && !mbar_wait_bounded(&full[s], ph)) {
           timed_out = true;
           if (lane == 0) atomicOr(&g_tc_status, SQ_DEV_TIMEOUT);
@@ -306,46 +325,61 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int h = 0; h < (SILU ? 2 : 1); ++h) {
           const uint8_t* codes = st + a.c_off + h * a.c_bytes;
           uint8_t* at = st + h * kTcStageA;
+          // one job = 16 code bytes of one row: 32 INT4 / 16 FP8 weights,
+          // i.e. 4 / 2 of the row's eight 16-byte fp16 chunks.  Per warp the
+          // code loads cover 512 contiguous bytes and each quarter-warp's
+          // chunk stores hit 8 distinct 16-byte bank groups (swizzle), so
+          // neither conflicts.
+          constexpr int kJobsPerRow = WK == 1 ? 2 : 4;
+          constexpr int kChunksPerJob = 8 / kJobsPerRow;
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            // 4 rows x 8 chunks per warp and pass: conflict-free reads and writes
-            const int job = j * 128 + ct;
-            const int row = job >> 3, c = job & 7;
-            uint4 out;
+          for (int job = ct; job < kTcBM * kJobsPerRow; job += 32 * TcConv<WK>::warps) {
+            const int row = job / kJobsPerRow, jp = job % kJobsPerRow;
+            const uint4 cw = *reinterpret_cast<const uint4*>(codes + row * (kTcBK * (WK == 1 ? 1 : 2) / 2) +
+                                                             jp * 16);
+            uint8_t* arow = at + row * 128;
             if constexpr (WK == 2) {
-              const uint2 cw = *reinterpret_cast<const uint2*>(codes + row * 64 + c * 8);
-              out.x = e4m3x2_to_f16x2(lo16(cw.x));
-              out.y = e4m3x2_to_f16x2(hi16(cw.x));
-              out.z = e4m3x2_to_f16x2(lo16(cw.y));
-              out.w = e4m3x2_to_f16x2(hi16(cw.y));
+              const uint32_t wv[4] = {cw.x, cw.y, cw.z, cw.w};
+#pragma unroll
+              for (int q = 0; q < 2; ++q) {
+                uint4 out;
+                out.x = e4m3x2_to_f16x2(lo16(wv[2 * q]));
+                out.y = e4m3x2_to_f16x2(hi16(wv[2 * q]));
+                out.z = e4m3x2_to_f16x2(lo16(wv[2 * q + 1]));
+                out.w = e4m3x2_to_f16x2(hi16(wv[2 * q + 1]));
+                const int c = jp * kChunksPerJob + q;
+                *reinterpret_cast<uint4*>(arow + ((c ^ (row & 7)) << 4)) = out;
+              }
             } else {
-              const uint32_t cw = *reinterpret_cast<const uint32_t*>(codes + row * 32 + c * 4);
-              uint32_t q[4];
-              int4x8_to_f16x2(cw, q);  // (k0,k4),(k1,k5),(k2,k6),(k3,k7)
-              const __half2 s2 = __half2half2(sc_cur[h][j]);
+              const __half2 s2 = __half2half2(sblk[(size_t)(h * kTcBM + row) * a.sc_ng + gi]);
               auto mul = [&](uint32_t v) {
                 const __half2 r = __hmul2(*reinterpret_cast<const __half2*>(&v), s2);
                 return *reinterpret_cast<const uint32_t*>(&r);
               };
-              out.x = mul(__byte_perm(q[0], q[1], 0x5410));  // (k0, k1)
-              out.y = mul(__byte_perm(q[2], q[3], 0x5410));  // (k2, k3)
-              out.z = mul(__byte_perm(q[0], q[1], 0x7632));  // (k4, k5)
-              out.w = mul(__byte_perm(q[2], q[3], 0x7632));  // (k6, k7)
+              const uint32_t wv[4] = {cw.x, cw.y, cw.z, cw.w};
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                uint32_t v[4];
+                int4x8_to_f16x2(wv[q], v);  // (k0,k4),(k1,k5),(k2,k6),(k3,k7)
+                uint4 out;
+                out.x = mul(__byte_perm(v[0], v[1], 0x5410));  // (k0, k1)
+                out.y = mul(__byte_perm(v[2], v[3], 0x5410));  // (k2, k3)
+                out.z = mul(__byte_perm(v[0], v[1], 0x7632));  // (k4, k5)
+                out.w = mul(__byte_perm(v[2], v[3], 0x7632));  // (k6, k7)
+                const int c = jp * kChunksPerJob + q;
+                *reinterpret_cast<uint4*>(arow + ((c ^ (row & 7)) << 4)) = out;
+              }
             }
-            *reinterpret_cast<uint4*>(at + row * 128 + ((c ^ (row & 7)) << 4)) = out;
           }
         }
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncwarp();
         if (lane == 0) mbar_arrive(&conv[s]);
-        if constexpr (WK == 1) {
-#pragma unroll
-          for (int h = 0; h < S2; ++h)
-#pragma unroll
-            for (int j = 0; j < 8; ++j) sc_cur[h][j] = sc_nxt[h][j];
-        }
       }
     }
+  }
+  if (warp >= 2 && warp < 6) {
+    // --------------------------------------------------------- epilogue
     if (!mbar_wait_bounded(accf, 0u)) {
       timed_out = true;
       if (lane == 0) atomicOr(&g_tc_status, SQ_DEV_TIMEOUT);
@@ -397,12 +431,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   if (S > 1) {
     cluster_sync();  // every partial tile is written
     if (warp >= 2) {
-      const int et = tid - 64;  // 0..127
+      const int et = tid - 64;  // 0 .. blockDim.x - 65
       const int rows = (kTcBM + S - 1) / S;  // this rank's rows [r0, r0 + nr)
       const int r0 = (int)rank * rows;
       const int nr = rows < kTcBM - r0 ? rows : kTcBM - r0;
       const float* part = reinterpret_cast<const float*>(stages);
-      for (int idx = et; idx < nr * a.M; idx += 128) {
+      for (int idx = et; idx < nr * a.M; idx += (int)blockDim.x - 64) {
         const int m = idx / nr, row = r0 + (idx - m * nr);
         const int64_t n = tile * kTcBM + row;
         float g = 0.0f, u = 0.0f;
@@ -517,7 +551,7 @@ static int tc_max_clusters(int S, size_t smem) {
   if (tc_prepare<WK, SILU>(smem) != cudaSuccess) return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)S, 1, 1);
-  cfg.blockDim = dim3(kTcThreads);
+  cfg.blockDim = dim3(TcConv<WK>::threads);
   cfg.dynamicSmemBytes = smem;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -549,16 +583,16 @@ static int tc_max_clusters(int S, size_t smem) {
 // CTA + 2 for the split reduction), at least 2 k-steps per CTA; ties keep
 // the smaller S.
 template <int WK, bool SILU>
-static int tc_pick_split(int64_t tiles, int ksteps, size_t smem) {
+static int tc_pick_split(int64_t tiles, int ksteps, size_t smem, int max_split) {
   if (WK != 1) {
     const int sms = device_sm_count();
     int S = 1;
-    while (S < kTcMaxSplit && tiles * S * 2 <= sms && ksteps >= 4 * S * 2) S <<= 1;
+    while (2 * S <= max_split && tiles * S * 2 <= sms && ksteps >= 4 * S * 2) S <<= 1;
     return S;
   }
   int best_s = 1;
   int64_t best = INT64_MAX;
-  for (int S = 1; S <= kTcMaxSplit && ksteps >= 2 * S; ++S) {
+  for (int S = 1; S <= max_split && ksteps >= 2 * S; ++S) {
     const int nc = tc_max_clusters<WK, SILU>(S, smem);
     if (nc <= 0) continue;
     const int64_t waves = (tiles + nc - 1) / nc;
@@ -577,11 +611,11 @@ static cudaError_t tc_launch_inst(const CUtensorMap& tw, const CUtensorMap& tx, 
   auto k = tc_linear_kernel<WK, SILU>;
   cudaError_t e = tc_prepare<WK, SILU>(smem);
   if (e != cudaSuccess) return e;
-  const int S = tc_pick_split<WK, SILU>(tiles, a.ksteps, smem);
+  const int S = tc_pick_split<WK, SILU>(tiles, a.ksteps, smem, a.max_split);
   a.splits = S;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)S, (unsigned)tiles, 1);
-  cfg.blockDim = dim3(kTcThreads);
+  cfg.blockDim = dim3(TcConv<WK>::threads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
   cudaLaunchAttribute attr[2];
@@ -653,12 +687,26 @@ cudaError_t launch_tc(int wk, const __half* x, const void* w, const void* scales
   const int64_t tiles = (N + kTcBM - 1) / kTcBM;
   a.part_stride = kTcBM + 4;
   const size_t part_bytes = (size_t)cols * a.part_stride * 4;
-  int ns = (int)((200 * 1024) / a.stage_bytes);
+  // INT4: room for a CTA's group scales, sized for an unsplit K range
+  // (a range of n stages touches at most (n - 1) / 2 + 2 groups)
+  a.sc_ng = 0;
+  size_t sc_bytes = 0;
+  if (wk == SQ_W_INT4) {
+    const int64_t G = K / 128;
+    const int64_t need = (a.ksteps - 1) / 2 + 2;
+    a.sc_ng = (int)(need < G ? need : G);
+    sc_bytes = (size_t)S2 * kTcBM * (size_t)a.sc_ng * 2;
+  }
+  int ns = (int)(((200 * 1024) - (int64_t)sc_bytes) / a.stage_bytes);
   if (ns > 8) ns = 8;
   if (ns < 2) ns = 2;
-  while ((size_t)ns * a.stage_bytes < part_bytes) ++ns;
   a.nstages = ns;
-  const size_t smem = 1024 + (size_t)ns * a.stage_bytes + (3 * ns + 2) * 8 + 16;
+  // split-K keeps its fp32 partial tile in the (then idle) stage memory;
+  // where that does not fit (very large M), K is not split
+  a.max_split = (size_t)ns * a.stage_bytes >= part_bytes ? kTcMaxSplit : 1;
+  const size_t fixed = (size_t)ns * a.stage_bytes + (3 * (size_t)ns + 2) * 8 + 16;
+  a.sc_off = (int)((fixed + 15) / 16 * 16);
+  const size_t smem = 1024 + (size_t)a.sc_off + sc_bytes;
   if (smem > 227 * 1024) return cudaErrorInvalidValue;
 #define SQ_TC_CASE(WK_)                                                                \
   if (wk == WK_) return silu ? tc_launch_inst<WK_, true>(tw, tx, a, tiles, smem, st)  \

@@ -180,3 +180,22 @@ def test_engine_choice_small_rows():
     assert sq.sq_linear_path(sq.SQ_W_INT4, 1, 256, 100, sq.SQ_EPI_NONE) == -1
     assert sq.sq_linear_path(sq.SQ_W_FP16, 0, 256, 256, sq.SQ_EPI_NONE) == -1
     assert sq.sq_linear_path(sq.SQ_W_FP16, 257, 256, 256, sq.SQ_EPI_NONE) == -1
+
+
+@pytest.mark.parametrize("kind", ["fp16", "int4", "fp8"])
+def test_tc_silu_largest_m(kind):
+    # M = 256 with the fused gate: the split-K partial tile would not fit in
+    # shared memory, so K stays unsplit
+    I, K, M = 320, 1536, 256
+    w = synth.weights_fp16(71, 2 * I, K)
+    x = synth.activations_fp16(72, M, K)
+    if kind == "fp16":
+        wd, sd, w64 = f16_to_dev(w), None, w.astype(np.float64)
+    else:
+        wd, sd, w64 = _quant_variant(kind, w)
+    wk = {"fp16": sq.SQ_W_FP16, "int4": sq.SQ_W_INT4, "fp8": sq.SQ_W_FP8}[kind]
+    y = torch.empty(M, I, dtype=torch.float16, device=dev())
+    sq.sq_linear_ex(wk, f16_to_dev(x), wd, sd, None, None, sq.SQ_EPI_SILU_GATE, y)
+    assert sq.sq_check() == 0
+    full = oracle.linear(x.astype(np.float64), w64)
+    assert_close(dev_to_f64(y), oracle.silu_gate(full[:, :I], full[:, I:]), f"{kind} silu M=256")
