@@ -97,6 +97,12 @@ def _load():
         "oq_sample": (ctypes.c_int, [P, P, I64, I64, P]),
         "oq_enum_sweep": (ctypes.c_int, [P, P, P, P, I64, I64, ctypes.c_int, ctypes.c_int,
                                          ctypes.c_int, P]),
+        "oq_exp_neg": (ctypes.c_float, [ctypes.c_float]),
+        "oq_exp_neg_array": (None, [P, I64, P]),
+        "oq_softmax_row": (ctypes.c_int, [P, I64, ctypes.c_float, P]),
+        "oq_accept_logits": (ctypes.c_int, [P, P, P, P, I64, I64, I64, ctypes.c_float, ctypes.c_int,
+                                            P, P]),
+        "oq_sample_logits": (ctypes.c_int, [P, P, I64, I64, ctypes.c_float, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -269,3 +275,54 @@ def enum_sweep(p, q, draft, u_fixed, pos: int, grid_bits: int = 24,
     if st != OK:
         raise ValueError(f"oq_enum_sweep status {st}")
     return hist
+
+
+# ---- probabilities from logits --------------------------------------------------
+
+def exp_neg(x) -> np.ndarray:
+    """e^x for x <= 0 by the oracle's fp32 Cody-Waite + Taylor-7 routine."""
+    xs = _c(np.atleast_1d(np.asarray(x, np.float32)), np.float32)
+    out = np.empty(xs.shape, np.float32)
+    _load().oq_exp_neg_array(_ptr(xs), xs.size, _ptr(out))
+    return out
+
+
+def softmax_row(z16, T: float = 1.0) -> np.ndarray:
+    """softmax(z / T) of one row of fp16 logits (bit patterns or float16)."""
+    za = _c(np.asarray(z16).view(np.uint16) if np.asarray(z16).dtype == np.float16
+            else z16, np.uint16)
+    p = np.empty(za.shape, np.float32)
+    st = _load().oq_softmax_row(_ptr(za), za.size, float(T), _ptr(p))
+    if st != OK:
+        raise ValueError("oq_softmax_row: bad arguments")
+    return p
+
+
+def accept_logits(zp, zq, draft, u, T: float = 1.0, mode: int = ACCEPT_SAMPLE):
+    """zp [B,K+1,V] fp16, zq [K,B,V] fp16 (None when K == 0), draft [B,K],
+    u [B,K+1] -> (status, n_accepted [B], tokens [B,K+1])."""
+    za = _c(np.asarray(zp).view(np.uint16), np.uint16)
+    B, K1, V = za.shape
+    K = K1 - 1
+    qa = None if zq is None else _c(np.asarray(zq).view(np.uint16), np.uint16)
+    da = _c(draft, np.int32).reshape(B, K)
+    ua = _c(u, np.float32).reshape(B, K1)
+    n = np.empty((B,), np.int32)
+    t = np.empty((B, K1), np.int32)
+    st = _load().oq_accept_logits(_ptr(za), _ptr(qa), _ptr(da), _ptr(ua), B, K, V, float(T), mode,
+                                  _ptr(n), _ptr(t))
+    if st == BAD_ARG:
+        raise ValueError("oq_accept_logits: bad arguments")
+    return st, n, t
+
+
+def sample_logits(z, u, T: float = 1.0):
+    """token[b] ~ softmax(z[b,:] / T) by the fixed-point inverse CDF."""
+    za = _c(np.asarray(z).view(np.uint16), np.uint16)
+    B, V = za.shape
+    ua = _c(u, np.float32).reshape(B)
+    t = np.empty((B,), np.int32)
+    st = _load().oq_sample_logits(_ptr(za), _ptr(ua), B, V, float(T), _ptr(t))
+    if st == BAD_ARG:
+        raise ValueError("oq_sample_logits: bad arguments")
+    return st, t

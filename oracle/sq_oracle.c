@@ -374,3 +374,94 @@ int oq_sample(const float* probs, const float* u, int64_t B, int64_t V,
   }
   return status;
 }
+
+/* ---- probabilities from logits ------------------------------------------ */
+
+float oq_exp_neg(float x) {
+  /* fp32 constants (exact hexadecimal values):
+   *   log2(e) rounded; ln 2 = LN2_HI + LN2_LO with LN2_HI holding 16
+   *   significant bits (so n * LN2_HI is exact for |n| < 256); 1/k! rounded. */
+  const float LOG2E = 0x1.715476p+0f;
+  const float LN2_HI = 0x1.62e4p-1f;
+  const float LN2_LO = 0x1.7f7d1cp-20f;
+  const float C2 = 0x1p-1f, C3 = 0x1.555556p-3f, C4 = 0x1.555556p-5f;
+  const float C5 = 0x1.111112p-7f, C6 = 0x1.6c16c2p-10f, C7 = 0x1.a01a02p-13f;
+  if (!(x > -104.0f)) return 0.0f;
+  const float n = rintf(x * LOG2E);
+  float r = fmaf(-n, LN2_HI, x);
+  r = fmaf(-n, LN2_LO, r);
+  float p = C7;
+  p = fmaf(p, r, C6);
+  p = fmaf(p, r, C5);
+  p = fmaf(p, r, C4);
+  p = fmaf(p, r, C3);
+  p = fmaf(p, r, C2);
+  p = fmaf(p, r, 1.0f);
+  p = fmaf(p, r, 1.0f);
+  const int ni = (int)n;
+  union { uint32_t u; float f; } sc;
+  if (ni >= -126) {
+    sc.u = (uint32_t)(ni + 127) << 23;
+    return p * sc.f;
+  }
+  sc.u = (uint32_t)(ni + 127 + 64) << 23;   /* 2^(n+64), normal */
+  const float t = p * sc.f;                 /* exact */
+  return t * 0x1p-64f;                      /* one rounding into the subnormals */
+}
+
+void oq_exp_neg_array(const float* x, int64_t n, float* out) {
+  for (int64_t i = 0; i < n; ++i) out[i] = oq_exp_neg(x[i]);
+}
+
+int oq_softmax_row(const uint16_t* z, int64_t V, float T, float* p) {
+  if (V < 1 || !(T > 0.0f) || !isfinite(T)) return OQ_BAD_ARG;
+  float m = -INFINITY;
+  for (int64_t v = 0; v < V; ++v) {
+    const float zv = (float)oq_f16_decode(z[v]);
+    if (!isfinite(zv)) return OQ_BAD_ARG;
+    if (zv > m) m = zv;
+  }
+  const float invT = 1.0f / T;
+  uint64_t S = 0;
+  for (int64_t v = 0; v < V; ++v) {
+    const float e = oq_exp_neg(((float)oq_f16_decode(z[v]) - m) * invT);
+    p[v] = e;                                      /* e_v for now */
+    S += (uint64_t)floor(ldexp((double)e, 40));    /* exact: e <= 1 */
+  }
+  const float s = (float)ldexp((double)S, -40);
+  for (int64_t v = 0; v < V; ++v) p[v] = p[v] / s;
+  return OQ_OK;
+}
+
+int oq_accept_logits(const uint16_t* zp, const uint16_t* zq, const int32_t* draft,
+                     const float* u, int64_t B, int64_t K, int64_t V, float T,
+                     int mode, int32_t* n_accepted, int32_t* tokens) {
+  if (B < 0 || K < 0 || V <= 0) return OQ_BAD_ARG;
+  if (K > 0 && zq == NULL) return OQ_BAD_ARG;
+  float* p = (float*)malloc((size_t)(B * (K + 1) * V + (K > 0 ? B * K * V : 0) + 1) * sizeof(float));
+  if (!p) return OQ_BAD_ARG;
+  float* q = p + B * (K + 1) * V;
+  int st = OQ_OK;
+  for (int64_t b = 0; b < B && st == OQ_OK; ++b) {
+    for (int64_t i = 0; i <= K && st == OQ_OK; ++i)
+      st = oq_softmax_row(zp + (b * (K + 1) + i) * V, V, T, p + (b * (K + 1) + i) * V);
+    for (int64_t i = 0; i < K && st == OQ_OK; ++i)  /* zq row of step i, sequence b */
+      st = oq_softmax_row(zq + (i * B + b) * V, V, T, q + (b * K + i) * V);
+  }
+  if (st == OQ_OK)
+    st = oq_accept(p, K > 0 ? q : NULL, draft, u, B, K, V, mode, n_accepted, tokens);
+  free(p);
+  return st;
+}
+
+int oq_sample_logits(const uint16_t* z, const float* u, int64_t B, int64_t V,
+                     float T, int32_t* tokens) {
+  if (B < 0 || V <= 0) return OQ_BAD_ARG;
+  float* p = (float*)malloc((size_t)(B * V + 1) * sizeof(float));
+  if (!p) return OQ_BAD_ARG;
+  int st = OQ_OK;
+  for (int64_t b = 0; b < B && st == OQ_OK; ++b) st = oq_softmax_row(z + b * V, V, T, p + b * V);
+  if (st == OQ_OK) st = oq_sample(p, u, B, V, tokens);
+  free(p);
+  return st;
+}

@@ -100,6 +100,37 @@ int oq_accept(const float* p, const float* q, const int32_t* draft,
 int oq_sample(const float* probs, const float* u, int64_t B, int64_t V,
               int32_t* tokens);
 
+/* ---- probabilities from logits (softmax with temperature) ------------------
+ * The paper's parents emit next-token distributions (Sec. III-D.2/3); a
+ * decoder's lm_head emits logits z, and p = softmax(z / T).  The paper fixes
+ * no arithmetic for it; the definition implemented here is exactly
+ * reproducible in IEEE fp32 on any machine:
+ *   m    = max_v z_v (fp16 logits, exact in fp32)
+ *   invT = 1 / T (fp32 division)
+ *   e_v  = exp_neg((z_v - m) * invT)        (fp32 subtract, then multiply)
+ *   S    = sum_v floor(e_v * 2^40)          (64-bit integer, order-free)
+ *   s    = (float)((double)S * 2^-40)
+ *   p_v  = e_v / s                          (fp32 division)
+ * exp_neg(x) for x <= 0: Cody-Waite reduction x = n ln2 + r (ln 2 split in
+ * a 16-bit head and a tail so n * head is exact), e^r by its degree-7
+ * Taylor polynomial in Horner form with fused multiply-adds, then the
+ * exact scaling by 2^n (through 2^(n+64) * 2^-64 below 2^-126); 0 for
+ * x <= -104 (below the smallest subnormal). */
+float oq_exp_neg(float x);
+void oq_exp_neg_array(const float* x, int64_t n, float* out);
+/* One row: z [V] fp16 bit patterns, T > 0 -> p [V].  OQ_BAD_ARG for V < 1,
+ * T not a positive finite number, or a non-finite logit. */
+int oq_softmax_row(const uint16_t* z, int64_t V, float T, float* p);
+/* Sec. III-D.4 from logits: zp [B,K+1,V] (target, position-major per
+ * sequence), zq [K,B,V] (draft, one [B,V] block per draft step); p and q
+ * rows by oq_softmax_row, then exactly oq_accept. */
+int oq_accept_logits(const uint16_t* zp, const uint16_t* zq, const int32_t* draft,
+                     const float* u, int64_t B, int64_t K, int64_t V, float T,
+                     int mode, int32_t* n_accepted, int32_t* tokens);
+/* Draft-side sampling from logits: token[b] ~ softmax(z[b,:] / T). */
+int oq_sample_logits(const uint16_t* z, const float* u, int64_t B, int64_t V,
+                     float T, int32_t* tokens);
+
 /* ---- exhaustive-enumeration harness (sq_enumerate.c) --------------------- */
 /* Runs oq_accept on one sequence 2^grid_bits times, with the uniform at
  * position `pos` set to m * 2^-grid_bits for every m, the others taken from
