@@ -71,6 +71,16 @@ def measured_peaks():
     return 6800.0, "fallback"
 
 
+def measured_tensor_peak():
+    """Sustained dense bf16 TFLOP/s (fp16 runs at the same tensor rate)."""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        if "bf16_tflops_sustained" in d:
+            return float(d["bf16_tflops_sustained"]), "measured sustained"
+    return 1700.0, "fallback sustained"
+
+
 class ClockSampler:
     """nvidia-smi samples (200 ms) of SM clock and throttle reasons."""
 
@@ -215,14 +225,22 @@ def cpu_oracle_prepare(shape, variant, B, K, layers=1, lm_rows=None, seed=0):
         items.append((n, k, silu, w16, q, xd, xv))
     sample_w = sum(n * k for n, k, *_ in items)
     total_w = shape.linear_params()
-    desc = (f"oracle (plain C, fp64, 1 thread) on {layers} of {shape.layers} layers + {lm_rows} of "
-            f"{shape.vocab} lm_head rows ({sample_w / 1e6:.1f}M of {total_w / 1e6:.0f}M weights: "
-            f"dequantise + {K} draft linears at M={Md} + 1 verify linear at M={Mv}) and the full "
-            f"accept over V={shape.vocab}; extrapolated to the whole step by weight count")
-    return {"items": items, "variant": variant, "K": K, "scale": total_w / sample_w, "desc": desc}
+    V = shape.vocab
+    # logits of one cycle (fp16) for the draft samples and the accept
+    zp = rng.normal(0, 2.0, (B, K + 1, V)).astype(np.float16)
+    zq = (np.transpose(zp[:, :K, :], (1, 0, 2)).astype(np.float32) +
+          rng.normal(0, 0.5, (K, B, V))).astype(np.float16)
+    u_draft = synth.uniforms(31, (K, B))
+    desc = (f"oracle (plain C, fp64 linears, 1 thread) on {layers} of {shape.layers} layers + "
+            f"{lm_rows} of {V} lm_head rows ({sample_w / 1e6:.1f}M of {total_w / 1e6:.0f}M weights: "
+            f"dequantise + {K} draft linears at M={Md} + 1 verify linear at M={Mv}), extrapolated "
+            f"to the whole step by weight count, plus the full {K} draft samples and the accept "
+            f"from logits over V={V}")
+    return {"items": items, "variant": variant, "K": K, "scale": total_w / sample_w, "desc": desc,
+            "zp": zp, "zq": zq, "u_draft": u_draft}
 
 
-def cpu_oracle_run(prep, p, q, draft, u):
+def cpu_oracle_run(prep, draft, u):
     """One timed oracle step on the prepared sample; returns (seconds of
     the full step extrapolated by weight count, seconds spent)."""
     import oracle
@@ -243,7 +261,9 @@ def cpu_oracle_run(prep, p, q, draft, u):
             oracle.silu_gate(yv[:, : n // 2], yv[:, n // 2:])
         t_lin += time.perf_counter() - t0
     t0 = time.perf_counter()
-    oracle.accept(p, q, draft, u, oracle.ACCEPT_SAMPLE)
+    for k in range(prep["K"]):
+        oracle.sample_logits(prep["zq"][k], prep["u_draft"][k])
+    oracle.accept_logits(prep["zp"], prep["zq"], draft, u, 1.0, oracle.ACCEPT_SAMPLE)
     t_acc = time.perf_counter() - t0
     return t_lin * prep["scale"] + t_acc, t_lin + t_acc
 
@@ -305,13 +325,29 @@ def main():
     if args.case:
         return run_case(args, stack, bd, bv, (tp, tq, td, tu, n_out, tok_out, ws), stream, peak_gbs)
 
-    def step():
-        for _ in range(K):
-            stk.run_pass(stack, args.draft, bd, stream)
-        stk.run_pass(stack, "fp16", bv, stream)
-        sq.sq_accept(tp, tq, td, tu, sq.SQ_ACCEPT_SAMPLE, n_out, tok_out, ws, stream)
+    # the cycle on its own logits: draft step k's lm_head writes zq[k] and a
+    # draft token is sampled from it; the verify pass's lm_head output is
+    # the target logits [B, K+1, V]; accept / resample runs on both (the
+    # probabilities are never written).  The linear stack has no embedding,
+    # so the sampled draft tokens are not fed back; the accept tests the
+    # block's synthetic draft tokens.
+    temperature = 1.0
+    zq = torch.empty(K, B, V, dtype=torch.float16, device=dev)
+    zp = bv.logits.view(B, K + 1, V)
+    u_draft = torch.from_numpy(synth.uniforms(31 + rank, (K, B))).to(dev)
+    samp = torch.empty(K, B, 1, dtype=torch.int32, device=dev)
+    ws_s = torch.zeros(sq.sq_accept_logits_workspace_bytes(B, 0, V), dtype=torch.uint8, device=dev)
+    ws_l = torch.zeros(sq.sq_accept_logits_workspace_bytes(B, K, V), dtype=torch.uint8, device=dev)
 
-    launches_per_step = (K + 1) * stack.launches_per_pass() + 1
+    def step():
+        for k in range(K):
+            stk.run_pass(stack, args.draft, bd, stream, logits=zq[k])
+            sq.sq_sample_logits(zq[k], u_draft[k], temperature, samp[k], ws_s, stream)
+        stk.run_pass(stack, "fp16", bv, stream)
+        sq.sq_accept_logits(zp, zq, td, tu, temperature, sq.SQ_ACCEPT_SAMPLE, n_out, tok_out, ws_l,
+                            stream)
+
+    launches_per_step = (K + 1) * stack.launches_per_pass() + 3 * K + 3
 
     def capture(fn):
         with torch.cuda.stream(stream):
@@ -364,17 +400,37 @@ def main():
         g_ver = pass_graph("fp16", bv)
         g_acc = capture(lambda: sq.sq_accept(tp, tq, td, tu, sq.SQ_ACCEPT_SAMPLE, n_out, tok_out, ws,
                                              stream))
+        g_accl = capture(lambda: sq.sq_accept_logits(zp, zq, td, tu, temperature, sq.SQ_ACCEPT_SAMPLE,
+                                                     n_out, tok_out, ws_l, stream))
+        g_smpl = capture(lambda: sq.sq_sample_logits(zq[0], u_draft[0], temperature, samp[0], ws_s,
+                                                     stream))
         t_draft = timed(g_draft, reps) / reps
         t_ver = timed(g_ver, reps) / reps
         t_acc = timed(g_acc, reps) / reps
+        t_accl = timed(g_accl, reps) / reps
+        t_smpl = timed(g_smpl, reps) / reps
         # the same passes as separate sq_linear_ex calls
         g_draft_u = capture(lambda: stk.run_pass_unchained(stack, args.draft, bd, stream))
         g_ver_u = capture(lambda: stk.run_pass_unchained(stack, "fp16", bv, stream))
         t_draft_u = timed(g_draft_u, reps) / reps
         t_ver_u = timed(g_ver_u, reps) / reps
+        # prefill of a 256-token prompt through the stack (tensor cores), the
+        # parent and the draft variant
+        bp = stk.PassBuffers(stack, 256, seed=17 + rank)
+        reps_pf = max(5, reps // 10)
+        g_pf16 = pass_graph("fp16", bp)
+        t_pf16 = timed(g_pf16, reps_pf) / reps_pf
+        g_pfd = pass_graph(args.draft, bp)
+        t_pfd = timed(g_pfd, reps_pf) / reps_pf
+        del g_pf16, g_pfd, bp
+    tensor_peak, tensor_peak_kind = measured_tensor_peak()
+    pf_flops = 2.0 * 256 * stack.params()
     draft_bytes = stack.weight_bytes(args.draft) + stack.activation_bytes(B)
     ver_bytes = stack.weight_bytes("fp16") + stack.activation_bytes(Mv)
     acc_bytes = B * (2 * V * 4 + 2 * K * 4)
+    # accept from logits: two statistics passes over the 2K+1 rows of fp16
+    # logits, then the correction rows (p and q) once more
+    accl_bytes = B * ((2 * K + 1) * V * 2 * 2 + 2 * V * 2)
 
     # ---- dominant kernel: the fused gate/up + SiLU linear (largest per-launch
     # weight matrix in the layers); all layers' launches of it in one graph
@@ -405,15 +461,14 @@ def main():
     if not args.no_e2e:
         h_xd = torch.empty_like(bd.x, device="cpu").pin_memory()
         h_xv = torch.empty_like(bv.x, device="cpu").pin_memory()
-        h_p = torch.from_numpy(p).pin_memory()
-        h_q = torch.from_numpy(q).pin_memory()
         h_d = torch.from_numpy(draft).pin_memory()
         h_u = torch.from_numpy(u).pin_memory()
+        h_ud = u_draft.cpu().pin_memory()
         h_xd.copy_(bd.x.cpu())
         h_xv.copy_(bv.x.cpu())
         h_n = torch.empty(B, dtype=torch.int32).pin_memory()
         h_t = torch.empty(B, K + 1, dtype=torch.int32).pin_memory()
-        h2d = sum(t.numel() * t.element_size() for t in (h_xd, h_xv, h_p, h_q, h_d, h_u))
+        h2d = sum(t.numel() * t.element_size() for t in (h_xd, h_xv, h_d, h_u, h_ud))
         d2h = h_n.numel() * 4 + h_t.numel() * 4
         e2e_steps = max(10, min(args.steps, 200))
 
@@ -421,10 +476,9 @@ def main():
             with torch.cuda.stream(stream):
                 bd.x.copy_(h_xd, non_blocking=True)
                 bv.x.copy_(h_xv, non_blocking=True)
-                tp.copy_(h_p, non_blocking=True)
-                tq.copy_(h_q, non_blocking=True)
                 td.copy_(h_d, non_blocking=True)
                 tu.copy_(h_u, non_blocking=True)
+                u_draft.copy_(h_ud, non_blocking=True)
                 g_step.replay()
                 h_n.copy_(n_out, non_blocking=True)
                 h_t.copy_(tok_out, non_blocking=True)
@@ -446,7 +500,7 @@ def main():
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         prep = cpu_oracle_prepare(shape, args.draft, B, K, layers=1)
-        runs = [cpu_oracle_run(prep, p, q, draft, u) for _ in range(3)]
+        runs = [cpu_oracle_run(prep, draft, u) for _ in range(3)]
         t_full = statistics.median(r[0] for r in runs)
         cpu = {"value": tokens_per_step / t_full, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": prep["desc"] + "; median of 3 runs",
@@ -476,13 +530,23 @@ def main():
         "breakdown": {
             "draft_pass_ms": 1e3 * t_draft, "draft_pass_gbs": draft_bytes / t_draft / 1e9,
             "verify_pass_ms": 1e3 * t_ver, "verify_pass_gbs": ver_bytes / t_ver / 1e9,
-            "accept_ms": 1e3 * t_acc, "accept_gbs": acc_bytes / t_acc / 1e9,
+            "accept_logits_ms": 1e3 * t_accl,
+            "accept_logits_gbs": accl_bytes / t_accl / 1e9,
+            "sample_logits_ms": 1e3 * t_smpl,
+            "accept_from_probabilities_ms": 1e3 * t_acc,
+            "accept_from_probabilities_gbs": acc_bytes / t_acc / 1e9,
             "draft_pass_unchained_ms": 1e3 * t_draft_u, "verify_pass_unchained_ms": 1e3 * t_ver_u,
             "draft_pass_frac_of_peak": draft_bytes / t_draft / 1e9 / peak_gbs,
             "verify_pass_frac_of_peak": ver_bytes / t_ver / 1e9 / peak_gbs,
             "fp16_gateup_silu_m%d_us" % Mv: 1e6 * t_gu16,
             "fp16_gateup_silu_gbs": gu16_bytes / t_gu16 / 1e9,
             "launches_per_pass": stack.launches_per_pass(),
+            "prefill_m256_fp16_ms": 1e3 * t_pf16,
+            "prefill_m256_fp16_tflops": pf_flops / t_pf16 / 1e12,
+            "prefill_m256_%s_ms" % args.draft: 1e3 * t_pfd,
+            "prefill_m256_%s_tflops" % args.draft: pf_flops / t_pfd / 1e12,
+            "prefill_tensor_peak_tflops": tensor_peak,
+            "prefill_tensor_peak_source": f"{tensor_peak_kind} (MEASURED_PEAKS.json bf16_tflops_sustained)",
             # the same step time with the paper's measured acceptance rates
             # (Table II), E[tokens per cycle] = (1 - a^(K+1)) / (1 - a)
             "projected_tokens_per_s_at_paper_alpha": {
@@ -573,7 +637,7 @@ def main_reference():
     desc = prep["desc"]
     times = []
     for i in range(args.warmup + args.steps):
-        t_full, _ = cpu_oracle_run(prep, p, q, draft, u)
+        t_full, _ = cpu_oracle_run(prep, draft, u)
         if i >= args.warmup:
             times.append(t_full)
     t = sum(times)

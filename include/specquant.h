@@ -74,6 +74,7 @@ typedef enum { SQ_ACCEPT_SAMPLE = 0, SQ_ACCEPT_GREEDY = 1 } sq_accept_mode;
 #define SQ_DEV_NO_MASS          0x4u  /* sq_accept/sq_sample: row w/o mass   */
 #define SQ_DEV_BAD_UNIFORM      0x8u  /* resampling uniform not in [0,1)     */
 #define SQ_DEV_TIMEOUT          0x10u /* a kernel gave up a bounded wait     */
+#define SQ_DEV_NONFINITE_LOGIT  0x20u /* a logit row held inf or NaN         */
 
 /* Thread-local text of the last error raised on this host thread. */
 SQ_API const char* sq_last_error(void);
@@ -234,6 +235,56 @@ SQ_API sq_status sq_accept(const float* p, const float* q, const int32_t* draft,
  * workspace rules, workspace size sq_accept_workspace_bytes(B, 0, V)). */
 SQ_API sq_status sq_sample(const float* probs, const float* u, int B, int64_t V, int32_t* tokens,
                     void* workspace, size_t ws_bytes, sq_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Sec. III-D.4 from logits: the same accept / reject / resample step, with
+ * the probabilities computed inside the library from the lm_head outputs
+ * instead of read from memory (no [B, K+1, V] fp32 array is written).
+ *
+ *   zp  fp16 [B, K+1, V]  target logits (row b (K+1) + i: sequence b,
+ *                         position i: the verify pass's lm_head output)
+ *   zq  fp16 [K, B, V]    draft logits (block i: the lm_head output of draft
+ *                         step i for all B sequences; NULL allowed when
+ *                         K == 0)
+ *   temperature T > 0 and finite.
+ *
+ * p_i = softmax(zp[b, i, :] / T), q_i = softmax(zq[i, b, :] / T), each row
+ * computed exactly as
+ *   m = max_v z_v,  invT = 1/T (fp32),  e_v = exp_neg((z_v - m) * invT),
+ *   S = sum_v floor(e_v * 2^40) (64-bit integer),  s = (float)(S * 2^-40),
+ *   p_v = e_v / s (fp32 division),
+ * where exp_neg(x) (x <= 0) is a Cody-Waite reduction by ln 2 (16-bit head
+ * plus tail) and a degree-7 Taylor polynomial evaluated with fused
+ * multiply-adds, scaled by 2^n, and 0 for x <= -104; every step is an IEEE
+ * fp32 operation rounded to nearest, so the probabilities are bit-identical
+ * to this definition.  Everything after that is sq_accept on these rows
+ * (both modes; greedy takes argmax p).  A sequence with a non-finite logit in
+ * any of its 2K+1 rows gets n_accepted = -1 and all tokens -1, and sets
+ * SQ_DEV_NONFINITE_LOGIT.  Pointers: zp, zq 2-byte aligned, the rest as for
+ * sq_accept.  workspace: sq_accept_logits_workspace_bytes(B, K, V) bytes,
+ * 16-byte aligned, zero-filled before first use (each call leaves it so);
+ * calls sharing a workspace must not overlap on the GPU. */
+SQ_API size_t sq_accept_logits_workspace_bytes(int B, int K, int64_t V);
+SQ_API sq_status sq_accept_logits(const void* zp, const void* zq, const int32_t* draft,
+                                  const float* u, int B, int K, int64_t V, float temperature,
+                                  sq_accept_mode mode, int32_t* n_accepted, int32_t* tokens,
+                                  void* workspace, size_t ws_bytes, sq_stream_t stream);
+/* Draft-side sampling from logits: token[b] ~ softmax(z[b, :] / T) with
+ * uniform u[b] (the K = 0 case of sq_accept_logits; z fp16 [B, V];
+ * workspace sq_accept_logits_workspace_bytes(B, 0, V)). */
+SQ_API sq_status sq_sample_logits(const void* z, const float* u, int B, int64_t V,
+                                  float temperature, int32_t* tokens, void* workspace,
+                                  size_t ws_bytes, sq_stream_t stream);
+
+/* The probabilities of sq_accept_logits on their own: p[r, :] =
+ * softmax(z[r, :] / T) for R rows of fp16 logits z [R, V] into fp32 p [R, V],
+ * by the definition above (bit-identical to it); a row holding a non-finite
+ * logit gives NaN and sets SQ_DEV_NONFINITE_LOGIT.  workspace:
+ * sq_softmax_workspace_bytes(R, V) bytes, 16-byte aligned, zero-filled
+ * before first use (each call leaves it so). */
+SQ_API size_t sq_softmax_workspace_bytes(int64_t R, int64_t V);
+SQ_API sq_status sq_softmax(const void* z, int64_t R, int64_t V, float temperature, float* p,
+                            void* workspace, size_t ws_bytes, sq_stream_t stream);
 
 /* ------------------------------------------------------------------------
  * sq_accept_noalloc: sq_accept without a caller workspace.  The paper has

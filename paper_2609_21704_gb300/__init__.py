@@ -27,6 +27,8 @@ __all__ = [
     "sq_quantized_bytes", "sq_quantize", "sq_linear_w4a16", "sq_linear_fp8", "sq_verify",
     "sq_linear_ex", "sq_accept_workspace_bytes", "sq_accept", "sq_sample", "sq_check",
     "sq_version", "sq_accept_noalloc", "sq_linear_path", "sq_linear_chain", "SqLinearOp",
+    "sq_accept_logits_workspace_bytes", "sq_accept_logits", "sq_sample_logits",
+    "sq_softmax_workspace_bytes", "sq_softmax",
     "EXPORTED_SYMBOLS",
 ]
 
@@ -36,6 +38,7 @@ SQ_ACCEPT_SAMPLE, SQ_ACCEPT_GREEDY = 0, 1
 SQ_EPI_NONE, SQ_EPI_SILU_GATE, SQ_EPI_RESIDUAL = 0, 1, 2
 SQ_W_FP16, SQ_W_INT4, SQ_W_FP8 = 0, 1, 2
 SQ_DEV_NONFINITE_WEIGHT, SQ_DEV_BAD_DRAFT_TOKEN, SQ_DEV_NO_MASS, SQ_DEV_BAD_UNIFORM = 1, 2, 4, 8
+SQ_DEV_TIMEOUT, SQ_DEV_NONFINITE_LOGIT = 0x10, 0x20
 
 _P = ctypes.c_void_p
 _I64 = ctypes.c_int64
@@ -58,6 +61,12 @@ _SIGS = {
     "sq_accept_noalloc": (_INT, [_P, _P, _P, _P, _INT, _INT, _I64, _INT, _P, _P, _P]),
     "sq_linear_path": (_INT, [_INT, _INT, _I64, _I64, _INT]),
     "sq_linear_chain": (_INT, [_P, _INT, _P]),
+    "sq_accept_logits_workspace_bytes": (_SIZE, [_INT, _INT, _I64]),
+    "sq_accept_logits": (_INT, [_P, _P, _P, _P, _INT, _INT, _I64, ctypes.c_float, _INT, _P, _P, _P,
+                                _SIZE, _P]),
+    "sq_sample_logits": (_INT, [_P, _P, _INT, _I64, ctypes.c_float, _P, _P, _SIZE, _P]),
+    "sq_softmax_workspace_bytes": (_SIZE, [_I64, _I64]),
+    "sq_softmax": (_INT, [_P, _I64, _I64, ctypes.c_float, _P, _P, _SIZE, _P]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGS)
 
@@ -182,6 +191,40 @@ def sq_verify(x, w16, bias, y, stream=None) -> None:
     N = y.shape[1]
     _check("sq_verify", load().sq_verify(_ptr(x), _ptr(w16), _ptr(bias), _ptr(y), M, N, K,
                                          _stream(stream)))
+
+
+def sq_accept_logits_workspace_bytes(B: int, K: int, V: int) -> int:
+    return int(load().sq_accept_logits_workspace_bytes(B, K, V))
+
+
+def sq_accept_logits(zp, zq, draft, u, temperature, mode, n_accepted, tokens, workspace,
+                     stream=None) -> None:
+    """zp fp16 [B,K+1,V] target logits, zq fp16 [K,B,V] draft logits (or None)."""
+    B, K1, V = zp.shape
+    _check("sq_accept_logits", load().sq_accept_logits(
+        _ptr(zp), _ptr(zq), _ptr(draft), _ptr(u), B, K1 - 1, V, float(temperature), mode,
+        _ptr(n_accepted), _ptr(tokens), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def sq_sample_logits(z, u, temperature, tokens, workspace, stream=None) -> None:
+    """token[b] ~ softmax(z[b] / T); z fp16 [B, V]."""
+    B, V = z.shape
+    _check("sq_sample_logits", load().sq_sample_logits(
+        _ptr(z), _ptr(u), B, V, float(temperature), _ptr(tokens), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def sq_softmax_workspace_bytes(R: int, V: int) -> int:
+    return int(load().sq_softmax_workspace_bytes(R, V))
+
+
+def sq_softmax(z, temperature, p, workspace, stream=None) -> None:
+    """p fp32 [R, V] = softmax(z / T) row by row; z fp16 [R, V]."""
+    R, V = z.shape
+    _check("sq_softmax", load().sq_softmax(_ptr(z), R, V, float(temperature), _ptr(p), _ptr(workspace),
+                                           workspace.numel() * workspace.element_size(),
+                                           _stream(stream)))
 
 
 def sq_accept_workspace_bytes(B: int, K: int, V: int) -> int:

@@ -30,17 +30,103 @@ __device__ unsigned int g_accept_status;
 // sq_accept_noalloc on a device reuses the same bytes.
 static __device__ __align__(256) unsigned char g_accept_scratch[kAcceptNoallocScratchBytes];
 
-// floor(r * 2^44) from the fp32 bits of r in [0, 1] (exact integer shifts).
-__device__ __forceinline__ unsigned long long fix44(float r) {
+// floor(r * 2^Q) from the fp32 bits of r in [0, 1] (exact integer shifts).
+template <int Q>
+__device__ __forceinline__ unsigned long long fixq(float r) {
   const uint32_t b = __float_as_uint(r);
   const uint32_t e = (b >> 23) & 0xffu;
   if ((b >> 31) || e == 0) return 0ull;  // zero, negative, or below 2^-126
   const unsigned long long mant = (unsigned long long)((b & 0x7fffffu) | 0x800000u);
-  const int sh = (int)e - 150 + 44;      // r = mant * 2^(e-150)
+  const int sh = (int)e - 150 + Q;       // r = mant * 2^(e-150)
   if (sh >= 0) return mant << sh;
   if (sh <= -64) return 0ull;
   return mant >> (-sh);
 }
+__device__ __forceinline__ unsigned long long fix44(float r) { return fixq<44>(r); }
+
+// ---- probabilities from logits (softmax with temperature) -----------------
+// e^x for x <= 0 in explicitly rounded fp32 operations: Cody-Waite reduction
+// x = n ln2 + r (ln 2 split into a head of 16 significant bits, so that
+// n * head is exact for |n| < 256, and a tail), e^r by its degree-7 Taylor
+// polynomial in Horner form with fused multiply-adds, then the exact
+// scaling by 2^n (through 2^(n+64) * 2^-64 below 2^-126: one rounding into
+// the subnormals); 0 for x <= -104 (below the smallest subnormal).  Only
+// _rn intrinsics are used, so nothing is contracted or reordered and the
+// bits follow from the definition.
+__device__ __forceinline__ float exp_neg(float x) {
+  if (!(x > -104.0f)) return 0.0f;
+  const float n = rintf(__fmul_rn(x, 0x1.715476p+0f));  // x log2(e), nearest integer
+  float r = __fmaf_rn(-n, 0x1.62e4p-1f, x);              // x - n ln2 (head)
+  r = __fmaf_rn(-n, 0x1.7f7d1cp-20f, r);                 // ... (tail)
+  float p = 0x1.a01a02p-13f;                             // 1/7!
+  p = __fmaf_rn(p, r, 0x1.6c16c2p-10f);                  // 1/6!
+  p = __fmaf_rn(p, r, 0x1.111112p-7f);                   // 1/5!
+  p = __fmaf_rn(p, r, 0x1.555556p-5f);                   // 1/4!
+  p = __fmaf_rn(p, r, 0x1.555556p-3f);                   // 1/3!
+  p = __fmaf_rn(p, r, 0.5f);
+  p = __fmaf_rn(p, r, 1.0f);
+  p = __fmaf_rn(p, r, 1.0f);
+  const int ni = (int)n;
+  if (ni >= -126) return __fmul_rn(p, __uint_as_float((uint32_t)(ni + 127) << 23));
+  return __fmul_rn(__fmul_rn(p, __uint_as_float((uint32_t)(ni + 127 + 64) << 23)), 0x1p-64f);
+}
+
+// p_v = e_v / s with e_v = exp_neg((z_v - m) * invT) (fp32 subtract, multiply,
+// divide, each rounded to nearest).
+__device__ __forceinline__ float logit_prob(__half z, float m, float invT, float s) {
+  return __fdiv_rn(exp_neg(__fmul_rn(__fsub_rn(__half2float(z), m), invT)), s);
+}
+
+// Probability sources of the accept kernel: rows of stored fp32
+// probabilities, or rows of fp16 logits with their softmax statistics.
+struct ProbRow {
+  const float* p;
+  __device__ __forceinline__ float operator()(int64_t v) const { return p[v]; }
+};
+struct ProbSrc {
+  const float* p;  // [B, K+1, V]
+  const float* q;  // [B, K, V] or null
+  int K;
+  int64_t V;
+  __device__ __forceinline__ ProbRow prow(int b, int i) const {
+    return ProbRow{p + ((int64_t)b * (K + 1) + i) * V};
+  }
+  __device__ __forceinline__ ProbRow qrow(int b, int i) const {
+    return ProbRow{q + ((int64_t)b * K + i) * V};
+  }
+  __device__ __forceinline__ bool has_q() const { return q != nullptr; }
+  __device__ __forceinline__ bool rows_ok(int, int) const { return true; }
+};
+struct LogitRow {
+  const __half* z;
+  float m, invT, s;
+  __device__ __forceinline__ float operator()(int64_t v) const { return logit_prob(z[v], m, invT, s); }
+};
+struct LogitSrc {
+  const __half* zp;  // [B, K+1, V]
+  const __half* zq;  // [K, B, V]
+  const float* m;    // row maxima: target rows b (K+1) + i, then draft rows B (K+1) + i B + b
+  const float* s;    // row normalisers, same order
+  float invT;
+  int B, K;
+  int64_t V;
+  __device__ __forceinline__ LogitRow prow(int b, int i) const {
+    const int64_t r = (int64_t)b * (K + 1) + i;
+    return LogitRow{zp + r * V, m[r], invT, s[r]};
+  }
+  __device__ __forceinline__ LogitRow qrow(int b, int i) const {
+    if (K == 0) return LogitRow{zp, 0.0f, 0.0f, 1.0f};  // no draft rows; never read
+    const int64_t r = (int64_t)i * B + b;
+    const int64_t rs = (int64_t)B * (K + 1) + r;
+    return LogitRow{zq + r * V, m[rs], invT, s[rs]};
+  }
+  __device__ __forceinline__ bool has_q() const { return K > 0; }
+  // row j of sequence b's 2K+1 rows has finite statistics (finite logits)
+  __device__ __forceinline__ bool rows_ok(int b, int j) const {
+    const int64_t r = j <= K ? (int64_t)b * (K + 1) + j : (int64_t)B * (K + 1) + (int64_t)(j - K - 1) * B + b;
+    return isfinite(m[r]) && isfinite(s[r]);
+  }
+};
 
 // floor(u * S) for u in [0, 1), exact (128-bit product of the 24-bit
 // significand and S, then a right shift).
@@ -80,7 +166,8 @@ __device__ __forceinline__ unsigned long long argmax_key(float v, int64_t idx) {
 
 constexpr int kAcceptThreads = 256;
 
-__global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a) {
+template <class Src>
+__global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a, Src src) {
   griddep_wait();
   griddep_launch_dependents();
   __shared__ unsigned long long red[kAcceptThreads / 32][17];
@@ -93,8 +180,6 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a) {
   const int b = (int)(bc / a.C), c = (int)(bc - (int64_t)b * a.C);
   const int K = a.K;
   const int64_t V = a.V;
-  const float* pb = a.p + (int64_t)b * (K + 1) * V;
-  const float* qb = a.q ? a.q + (int64_t)b * K * V : nullptr;
   const int32_t* xb = a.draft + (int64_t)b * K;
   const float* ub = a.u + (int64_t)b * (K + 1);
   const int64_t v0 = (int64_t)c * a.chunk;
@@ -104,18 +189,22 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a) {
   // ---- validity and (sampling) the accept tests, evaluated by warp 0
   if (warp == 0) {
     bool bad = false, acc = true;
+    // finite statistics for the sequence's rows (logits only)
+    bool rows_bad = false;
+    for (int j = lane; j <= 2 * K; j += 32) rows_bad |= !src.rows_ok(b, j);
+    const unsigned rows_mask = __ballot_sync(0xffffffffu, rows_bad);
     if (lane < K) {
       const int32_t x = xb[lane];
       bad = (x < 0 || (int64_t)x >= V);
-      if (!bad && a.mode == SQ_ACCEPT_SAMPLE)
-        acc = (double)ub[lane] * (double)qb[(int64_t)lane * V + x] < (double)pb[(int64_t)lane * V + x];
+      if (!bad && !rows_mask && a.mode == SQ_ACCEPT_SAMPLE)
+        acc = (double)ub[lane] * (double)src.qrow(b, lane)(x) < (double)src.prow(b, lane)(x);
     }
     const float uk = ub[K];
     const bool bad_u = !(uk >= 0.0f && uk < 1.0f);
     const unsigned bad_mask = __ballot_sync(0xffffffffu, bad);
     const unsigned rej_mask = __ballot_sync(0xffffffffu, lane < K && !acc);
     if (lane == 0) {
-      s_valid = (bad_mask == 0u) && !bad_u;
+      s_valid = (bad_mask == 0u) && !bad_u && !rows_mask;
       s_n = rej_mask ? (__ffs(rej_mask) - 1) : K;
       if (c == 0 && bad_mask) atomicOr(&g_accept_status, SQ_DEV_BAD_DRAFT_TOKEN);
       if (c == 0 && bad_u) atomicOr(&g_accept_status, SQ_DEV_BAD_UNIFORM);
@@ -126,13 +215,14 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a) {
 
   // ---- chunk partials
   if (a.mode == SQ_ACCEPT_SAMPLE) {
-    const float* pn = pb + (int64_t)n * V;
-    const float* qn = (n < K) ? qb + (int64_t)n * V : nullptr;
+    const auto pn = src.prow(b, n);
+    const bool use_q = n < K;
+    const auto qn = src.qrow(b, use_q ? n : 0);
     unsigned long long sr = 0, sp = 0;
     for (int64_t v = v0 + tid; v < v1; v += kAcceptThreads) {
-      const float pv = pn[v];
-      if (qn) {
-        const float d = pv - qn[v];
+      const float pv = pn(v);
+      if (use_q) {
+        const float d = pv - qn(v);
         sr += fix44(d > 0.0f ? d : 0.0f);
         sp += fix44(pv);
       } else {
@@ -158,10 +248,10 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a) {
   } else {
     // greedy: per position i, the maximum key over the chunk
     for (int i = 0; i <= K; ++i) {
-      const float* pi = pb + (int64_t)i * V;
+      const auto pi = src.prow(b, i);
       unsigned long long best = 0;
       for (int64_t v = v0 + tid; v < v1; v += kAcceptThreads) {
-        const unsigned long long k = argmax_key(pi[v], v);
+        const unsigned long long k = argmax_key(pi(v), v);
         best = k > best ? k : best;
       }
       best = warp_max_u64(best);
@@ -243,8 +333,9 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a) {
   }
   __syncthreads();
   if (s_valid) {
-    const float* pn = pb + (int64_t)n * V;
-    const float* qn = (n < K && !s_use_p) ? qb + (int64_t)n * V : nullptr;
+    const auto pn = src.prow(b, n);
+    const bool use_q = n < K && !s_use_p;
+    const auto qn = src.qrow(b, use_q ? n : 0);
     const int64_t w0 = (int64_t)s_chunk * a.chunk;
     const int64_t w1 = w0 + a.chunk < V ? w0 + a.chunk : V;
     const unsigned long long T = s_T;
@@ -253,9 +344,9 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a) {
       const int64_t v = base + tid;
       unsigned long long R = 0;
       if (v < w1) {
-        const float pv = pn[v];
-        if (qn) {
-          const float d = pv - qn[v];
+        const float pv = pn(v);
+        if (use_q) {
+          const float d = pv - qn(v);
           R = fix44(d > 0.0f ? d : 0.0f);
         } else {
           R = fix44(pv);
@@ -304,7 +395,177 @@ size_t accept_workspace_bytes(int B, int K, int64_t V) {
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t st) {
   if (a.B == 0) return cudaSuccess;
   const int64_t blocks = (int64_t)a.B * a.C;
-  return launch_pdl(accept_kernel, dim3((unsigned)blocks), dim3(kAcceptThreads), 0, st, a);
+  ProbSrc src{a.p, a.q, a.K, a.V};
+  return launch_pdl(accept_kernel<ProbSrc>, dim3((unsigned)blocks), dim3(kAcceptThreads), 0, st, a,
+                    src);
+}
+
+// ---- softmax statistics of logit rows --------------------------------------
+// One CTA per (row, chunk of kSoftmaxChunk entries).  Pass 1: the row
+// maximum (a NaN marks a row holding a non-finite logit); pass 2: the
+// fixed-point normaliser S = sum_v floor(e_v 2^40) and s = float(S 2^-40).
+// The last CTA of a row (atomic ticket, counter left at zero) combines the
+// chunk partials; max and integer sums do not depend on their order.
+__device__ __forceinline__ const __half* softmax_row_ptr(const SoftmaxArgs& a, int64_t r) {
+  return r < a.rp ? a.zp + r * a.V : a.zq + (r - a.rp) * a.V;
+}
+
+__global__ void __launch_bounds__(kAcceptThreads) softmax_max_kernel(SoftmaxArgs a) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ float red[kAcceptThreads / 32];
+  __shared__ int red_bad[kAcceptThreads / 32];
+  __shared__ int s_last;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t r = blockIdx.x / a.C;
+  const int c = (int)(blockIdx.x - r * a.C);
+  const __half* z = softmax_row_ptr(a, r);
+  const int64_t v0 = (int64_t)c * kSoftmaxChunk;
+  const int64_t v1 = v0 + kSoftmaxChunk < a.V ? v0 + kSoftmaxChunk : a.V;
+  float mx = -INFINITY;
+  int bad = 0;
+  for (int64_t v = v0 + tid; v < v1; v += kAcceptThreads) {
+    const float f = __half2float(z[v]);
+    bad |= !isfinite(f);
+    mx = fmaxf(mx, f);
+  }
+  mx = warp_max(mx);
+  bad = __any_sync(0xffffffffu, bad);
+  if (lane == 0) {
+    red[warp] = mx;
+    red_bad[warp] = bad;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    float m = -INFINITY;
+    int any_bad = 0;
+    for (int w = 0; w < kAcceptThreads / 32; ++w) {
+      m = fmaxf(m, red[w]);
+      any_bad |= red_bad[w];
+    }
+    a.pmax[r * a.C + c] = any_bad ? __int_as_float(0x7fc00000) : m;
+    __threadfence();
+    s_last = atomicAdd(&a.counter[r], 1u) == (unsigned)(a.C - 1);
+  }
+  __syncthreads();
+  if (tid == 0 && s_last) {
+    __threadfence();
+    float m = -INFINITY;
+    bool nan = false;
+    for (int cc = 0; cc < a.C; ++cc) {
+      const float pm = __ldcg(a.pmax + r * a.C + cc);
+      nan |= isnan(pm);
+      m = fmaxf(m, pm);
+    }
+    if (nan) {
+      m = __int_as_float(0x7fc00000);
+      atomicOr(&g_accept_status, SQ_DEV_NONFINITE_LOGIT);
+    }
+    a.m[r] = m;
+    a.counter[r] = 0u;
+  }
+}
+
+__global__ void __launch_bounds__(kAcceptThreads) softmax_sum_kernel(SoftmaxArgs a) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ unsigned long long red[kAcceptThreads / 32];
+  __shared__ int s_last;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t r = blockIdx.x / a.C;
+  const int c = (int)(blockIdx.x - r * a.C);
+  const __half* z = softmax_row_ptr(a, r);
+  const int64_t v0 = (int64_t)c * kSoftmaxChunk;
+  const int64_t v1 = v0 + kSoftmaxChunk < a.V ? v0 + kSoftmaxChunk : a.V;
+  const float m = a.m[r];
+  unsigned long long acc = 0;
+  if (isfinite(m))
+    for (int64_t v = v0 + tid; v < v1; v += kAcceptThreads)
+      acc += fixq<40>(exp_neg(__fmul_rn(__fsub_rn(__half2float(z[v]), m), a.invT)));
+  acc = warp_sum_u64(acc);
+  if (lane == 0) red[warp] = acc;
+  __syncthreads();
+  if (tid == 0) {
+    unsigned long long t = 0;
+    for (int w = 0; w < kAcceptThreads / 32; ++w) t += red[w];
+    a.psum[r * a.C + c] = t;
+    __threadfence();
+    s_last = atomicAdd(&a.counter[r], 1u) == (unsigned)(a.C - 1);
+  }
+  __syncthreads();
+  if (tid == 0 && s_last) {
+    __threadfence();
+    unsigned long long S = 0;
+    for (int cc = 0; cc < a.C; ++cc) S += __ldcg(a.psum + r * a.C + cc);
+    a.s[r] = isfinite(m) ? __double2float_rn(__ull2double_rn(S) * 0x1p-40)
+                         : __int_as_float(0x7fc00000);
+    a.counter[r] = 0u;
+  }
+}
+
+cudaError_t launch_accept_logits(const AcceptArgs& a, const SoftmaxArgs& sa, cudaStream_t st) {
+  if (a.B == 0) return cudaSuccess;
+  const int64_t sblocks = sa.rows * sa.C;
+  cudaError_t e = launch_pdl(softmax_max_kernel, dim3((unsigned)sblocks), dim3(kAcceptThreads), 0, st, sa);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(softmax_sum_kernel, dim3((unsigned)sblocks), dim3(kAcceptThreads), 0, st, sa);
+  if (e != cudaSuccess) return e;
+  LogitSrc src{sa.zp, sa.zq, sa.m, sa.s, sa.invT, a.B, a.K, a.V};
+  const int64_t blocks = (int64_t)a.B * a.C;
+  return launch_pdl(accept_kernel<LogitSrc>, dim3((unsigned)blocks), dim3(kAcceptThreads), 0, st, a,
+                    src);
+}
+
+size_t softmax_rows_workspace_bytes(int64_t rows, int64_t V) {
+  if (rows < 0 || V <= 0) return 0;
+  const int64_t C = (V + kSoftmaxChunk - 1) / kSoftmaxChunk;
+  auto up16 = [](size_t x) { return (x + 15u) & ~(size_t)15u; };
+  return up16((size_t)rows * 4u) * 3u + up16((size_t)rows * (size_t)C * 4u) +
+         up16((size_t)rows * (size_t)C * 8u);
+}
+
+size_t softmax_workspace_bytes(int B, int K, int64_t V) {
+  if (B < 0 || K < 0) return 0;
+  return softmax_rows_workspace_bytes((int64_t)B * (K + 1) + (int64_t)B * K, V);
+}
+
+void softmax_layout(SoftmaxArgs& sa, void* ws) {
+  auto up16 = [](size_t x) { return (x + 15u) & ~(size_t)15u; };
+  char* sw = reinterpret_cast<char*>(ws);
+  sa.C = (int)((sa.V + kSoftmaxChunk - 1) / kSoftmaxChunk);
+  const size_t rows4 = up16((size_t)sa.rows * 4u);
+  sa.counter = reinterpret_cast<unsigned int*>(sw);
+  sa.m = reinterpret_cast<float*>(sw + rows4);
+  sa.s = reinterpret_cast<float*>(sw + 2 * rows4);
+  sa.pmax = reinterpret_cast<float*>(sw + 3 * rows4);
+  sa.psum = reinterpret_cast<unsigned long long*>(sw + 3 * rows4 + up16((size_t)sa.rows * sa.C * 4u));
+}
+
+// p[r, v] from the row statistics (the same expression the accept kernel
+// evaluates); NaN for a row holding a non-finite logit.
+__global__ void __launch_bounds__(kAcceptThreads) softmax_write_kernel(SoftmaxArgs a, float* p) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int64_t r = blockIdx.x / a.C;
+  const int c = (int)(blockIdx.x - r * a.C);
+  const __half* z = softmax_row_ptr(a, r);
+  const int64_t v0 = (int64_t)c * kSoftmaxChunk;
+  const int64_t v1 = v0 + kSoftmaxChunk < a.V ? v0 + kSoftmaxChunk : a.V;
+  const float m = a.m[r], sc = a.s[r];
+  const bool ok = isfinite(m) && isfinite(sc);
+  float* pr = p + r * a.V;
+  for (int64_t v = v0 + threadIdx.x; v < v1; v += kAcceptThreads)
+    pr[v] = ok ? logit_prob(z[v], m, a.invT, sc) : __int_as_float(0x7fc00000);
+}
+
+cudaError_t launch_softmax(const SoftmaxArgs& sa, float* p, cudaStream_t st) {
+  if (sa.rows == 0) return cudaSuccess;
+  const int64_t sblocks = sa.rows * sa.C;
+  cudaError_t e = launch_pdl(softmax_max_kernel, dim3((unsigned)sblocks), dim3(kAcceptThreads), 0, st, sa);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(softmax_sum_kernel, dim3((unsigned)sblocks), dim3(kAcceptThreads), 0, st, sa);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(softmax_write_kernel, dim3((unsigned)sblocks), dim3(kAcceptThreads), 0, st, sa, p);
 }
 
 // Device address of g_accept_scratch for the current device.  In host code

@@ -5,6 +5,7 @@
 #include <stdio.h>
 #include <stdlib.h>
 
+#include <cmath>
 #include <string>
 
 #include "sq_internal.h"
@@ -436,6 +437,111 @@ sq_status sq_sample(const float* probs, const float* u, int B, int64_t V, int32_
                     void* workspace, size_t ws_bytes, sq_stream_t stream) {
   return accept_common("sq_sample", probs, nullptr, nullptr, u, B, 0, V, SQ_ACCEPT_SAMPLE, nullptr,
                        tokens, workspace, ws_bytes, stream);
+}
+
+size_t sq_accept_logits_workspace_bytes(int B, int K, int64_t V) {
+  const size_t acc = accept_workspace_bytes(B, K, V);
+  const size_t sm = softmax_workspace_bytes(B, K, V);
+  if (acc == 0 || sm == 0) return 0;
+  return ((acc + 15u) & ~(size_t)15u) + sm;
+}
+
+static sq_status accept_logits_common(const char* who, const void* zp, const void* zq,
+                                      const int32_t* draft, const float* u, int B, int K, int64_t V,
+                                      float temperature, int mode, int32_t* n_accepted,
+                                      int32_t* tokens, void* workspace, size_t ws_bytes,
+                                      sq_stream_t stream) {
+  if (mode != SQ_ACCEPT_SAMPLE && mode != SQ_ACCEPT_GREEDY)
+    return fail(SQ_ERR_INVALID_ARG, "%s: unknown mode %d", who, mode);
+  if (B < 0 || K < 0 || K > 16 || V < 1 || V >= ((int64_t)1 << 20))
+    return fail(SQ_ERR_SHAPE, "%s: need B >= 0, 0 <= K <= 16, 1 <= V < 2^20 (B=%d K=%d V=%lld)", who, B,
+                K, (long long)V);
+  if (!(temperature > 0.0f) || !std::isfinite(temperature))
+    return fail(SQ_ERR_INVALID_ARG, "%s: temperature must be positive and finite", who);
+  if (B == 0) return SQ_OK;
+  if (!zp || !u || !tokens || (K > 0 && (!draft || !zq)))
+    return fail(SQ_ERR_INVALID_ARG, "%s: NULL logits, u, draft or tokens", who);
+  if (!aligned(zp, 2) || (zq && !aligned(zq, 2)) || !aligned(u, 4) || (draft && !aligned(draft, 4)) ||
+      !aligned(tokens, 4) || (n_accepted && !aligned(n_accepted, 4)))
+    return fail(SQ_ERR_ALIGN, "%s: logits must be 2-byte, other pointers 4-byte aligned", who);
+  const size_t need = sq_accept_logits_workspace_bytes(B, K, V);
+  if (!workspace || ws_bytes < need)
+    return fail(SQ_ERR_WORKSPACE, "%s: workspace %zu bytes < %zu required", who, ws_bytes, need);
+  if (!aligned(workspace, 16)) return fail(SQ_ERR_ALIGN, "%s: workspace must be 16-byte aligned", who);
+  auto up16 = [](size_t x) { return (x + 15u) & ~(size_t)15u; };
+  char* ws = reinterpret_cast<char*>(workspace);
+  AcceptArgs a = {};
+  a.draft = draft;
+  a.u = u;
+  a.B = B;
+  a.K = K;
+  a.V = V;
+  a.mode = mode;
+  a.n_out = n_accepted;
+  a.tok_out = tokens;
+  const size_t ctr = up16((size_t)B * 4u);
+  a.counter = reinterpret_cast<unsigned int*>(ws);
+  a.part = reinterpret_cast<unsigned long long*>(ws + ctr);
+  a.C = (int)((V + kAcceptChunk - 1) / kAcceptChunk);
+  a.chunk = kAcceptChunk;
+  a.slots = K + 1 > 2 ? K + 1 : 2;
+  // softmax statistics after the accept workspace
+  SoftmaxArgs sa = {};
+  sa.zp = reinterpret_cast<const __half*>(zp);
+  sa.zq = K > 0 ? reinterpret_cast<const __half*>(zq) : nullptr;
+  sa.rp = (int64_t)B * (K + 1);
+  sa.rows = sa.rp + (int64_t)B * K;
+  sa.V = V;
+  sa.invT = 1.0f / temperature;
+  softmax_layout(sa, ws + up16(accept_workspace_bytes(B, K, V)));
+  cudaError_t e = launch_accept_logits(a, sa, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_accept_logits: launch");
+  return SQ_OK;
+}
+
+sq_status sq_accept_logits(const void* zp, const void* zq, const int32_t* draft, const float* u, int B,
+                           int K, int64_t V, float temperature, sq_accept_mode mode,
+                           int32_t* n_accepted, int32_t* tokens, void* workspace, size_t ws_bytes,
+                           sq_stream_t stream) {
+  if (!n_accepted && B > 0) return fail(SQ_ERR_INVALID_ARG, "sq_accept_logits: NULL n_accepted");
+  return accept_logits_common("sq_accept_logits", zp, zq, draft, u, B, K, V, temperature, (int)mode,
+                              n_accepted, tokens, workspace, ws_bytes, stream);
+}
+
+sq_status sq_sample_logits(const void* z, const float* u, int B, int64_t V, float temperature,
+                           int32_t* tokens, void* workspace, size_t ws_bytes, sq_stream_t stream) {
+  return accept_logits_common("sq_sample_logits", z, nullptr, nullptr, u, B, 0, V, temperature,
+                              SQ_ACCEPT_SAMPLE, nullptr, tokens, workspace, ws_bytes, stream);
+}
+
+size_t sq_softmax_workspace_bytes(int64_t R, int64_t V) { return softmax_rows_workspace_bytes(R, V); }
+
+sq_status sq_softmax(const void* z, int64_t R, int64_t V, float temperature, float* p, void* workspace,
+                     size_t ws_bytes, sq_stream_t stream) {
+  if (R < 0 || V < 1 || V >= ((int64_t)1 << 20))
+    return fail(SQ_ERR_SHAPE, "sq_softmax: need R >= 0, 1 <= V < 2^20 (R=%lld V=%lld)", (long long)R,
+                (long long)V);
+  if (!(temperature > 0.0f) || !std::isfinite(temperature))
+    return fail(SQ_ERR_INVALID_ARG, "sq_softmax: temperature must be positive and finite");
+  if (R == 0) return SQ_OK;
+  if (!z || !p) return fail(SQ_ERR_INVALID_ARG, "sq_softmax: NULL z or p");
+  if (!aligned(z, 2) || !aligned(p, 4))
+    return fail(SQ_ERR_ALIGN, "sq_softmax: z must be 2-byte, p 4-byte aligned");
+  const size_t need = softmax_rows_workspace_bytes(R, V);
+  if (!workspace || ws_bytes < need)
+    return fail(SQ_ERR_WORKSPACE, "sq_softmax: workspace %zu bytes < %zu required", ws_bytes, need);
+  if (!aligned(workspace, 16)) return fail(SQ_ERR_ALIGN, "sq_softmax: workspace must be 16-byte aligned");
+  SoftmaxArgs sa = {};
+  sa.zp = reinterpret_cast<const __half*>(z);
+  sa.zq = nullptr;
+  sa.rp = R;
+  sa.rows = R;
+  sa.V = V;
+  sa.invT = 1.0f / temperature;
+  softmax_layout(sa, workspace);
+  cudaError_t e = launch_softmax(sa, p, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_softmax: launch");
+  return SQ_OK;
 }
 
 // Same step as sq_accept for callers that cannot allocate device memory:

@@ -105,6 +105,30 @@ size_t accept_workspace_bytes(int B, int K, int64_t V);
 constexpr size_t kAcceptNoallocScratchBytes = (size_t)1 << 20;
 cudaError_t accept_noalloc_scratch(void** ptr);
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t st);
+
+// Softmax statistics of the logit rows of one accept-from-logits call:
+// target rows zp [rp = B (K+1), V], then draft rows zq [K B, V].
+constexpr int kSoftmaxChunk = 8192;
+struct SoftmaxArgs {
+  const __half* zp;
+  const __half* zq;
+  int64_t rp;                // target rows
+  int64_t rows;              // target + draft rows
+  int64_t V;
+  float invT;                // 1 / temperature (fp32)
+  int C;                     // chunks per row
+  float* m;                  // [rows] row maxima
+  float* s;                  // [rows] normalisers
+  float* pmax;               // [rows * C]
+  unsigned long long* psum;  // [rows * C]
+  unsigned int* counter;     // [rows], zero on entry, left zero
+};
+size_t softmax_rows_workspace_bytes(int64_t rows, int64_t V);
+size_t softmax_workspace_bytes(int B, int K, int64_t V);
+// Points sa's counter / m / s / partial arrays into ws (sa.rows, sa.V set).
+void softmax_layout(SoftmaxArgs& sa, void* ws);
+cudaError_t launch_accept_logits(const AcceptArgs& a, const SoftmaxArgs& sa, cudaStream_t st);
+cudaError_t launch_softmax(const SoftmaxArgs& sa, float* p, cudaStream_t st);
 cudaError_t take_accept_status(uint32_t* bits);
 
 }  // namespace sq

@@ -138,8 +138,9 @@ class PassBuffers:
         self.attn = self.qkv.view(-1)[: M * sh.q_out].view(M, sh.q_out)
 
 
-def pass_ops(stack: LinearStack, variant: str, b: PassBuffers):
-    """The linear calls of one pass in decoder order, as sq_linear_chain ops."""
+def pass_ops(stack: LinearStack, variant: str, b: PassBuffers, logits=None):
+    """The linear calls of one pass in decoder order, as sq_linear_chain ops;
+    `logits` (fp16 [M, vocab]) replaces b.logits as the lm_head output."""
     wk = WKIND[variant]
     ops = []
     for layer in stack.layers:
@@ -149,18 +150,20 @@ def pass_ops(stack: LinearStack, variant: str, b: PassBuffers):
         ops.append((wk, b.x, *gu.weight(variant), None, None, SQ_EPI_SILU_GATE, b.h))
         ops.append((wk, b.h, *down.weight(variant), None, None, SQ_EPI_NONE, b.d))
     if stack.lm_head is not None:
-        ops.append((wk, b.x, *stack.lm_head.weight(variant), None, None, SQ_EPI_NONE, b.logits))
+        ops.append((wk, b.x, *stack.lm_head.weight(variant), None, None, SQ_EPI_NONE,
+                    b.logits if logits is None else logits))
     return ops
 
 
-def run_pass(stack: LinearStack, variant: str, b: PassBuffers, stream=None) -> None:
+def run_pass(stack: LinearStack, variant: str, b: PassBuffers, stream=None, logits=None) -> None:
     """One draft (variant int4/fp8) or verify (fp16, or fp8) pass: every
     projection of every layer plus lm_head, in decoder order, as one
     sq_linear_chain call."""
-    sq_linear_chain(pass_ops(stack, variant, b), stream)
+    sq_linear_chain(pass_ops(stack, variant, b, logits), stream)
 
 
-def run_pass_unchained(stack: LinearStack, variant: str, b: PassBuffers, stream=None) -> None:
+def run_pass_unchained(stack: LinearStack, variant: str, b: PassBuffers, stream=None,
+                       logits=None) -> None:
     """The same pass as separate sq_linear_ex calls."""
-    for (wk, x, w, s, bias, res, epi, y) in pass_ops(stack, variant, b):
+    for (wk, x, w, s, bias, res, epi, y) in pass_ops(stack, variant, b, logits):
         sq_linear_ex(wk, x, w, s, bias, res, epi, y, stream)
