@@ -79,9 +79,22 @@ __device__ __forceinline__ float logit_prob(__half z, float m, float invT, float
 
 // Probability sources of the accept kernel: rows of stored fp32
 // probabilities, or rows of fp16 logits with their softmax statistics.
+// Each row type reads one entry, or the 8 entries [v, v + 8) (those at or
+// past vend read as 0) with vector loads where the addresses allow.
 struct ProbRow {
   const float* p;
   __device__ __forceinline__ float operator()(int64_t v) const { return p[v]; }
+  __device__ __forceinline__ void load8(int64_t v, int64_t vend, float out[8]) const {
+    if (v + 8 <= vend && ((reinterpret_cast<uintptr_t>(p + v) & 15u) == 0)) {
+      const float4 a = *reinterpret_cast<const float4*>(p + v);
+      const float4 b = *reinterpret_cast<const float4*>(p + v + 4);
+      out[0] = a.x; out[1] = a.y; out[2] = a.z; out[3] = a.w;
+      out[4] = b.x; out[5] = b.y; out[6] = b.z; out[7] = b.w;
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) out[j] = v + j < vend ? p[v + j] : 0.0f;
+    }
+  }
 };
 struct ProbSrc {
   const float* p;  // [B, K+1, V]
@@ -101,7 +114,43 @@ struct LogitRow {
   const __half* z;
   float m, invT, s;
   __device__ __forceinline__ float operator()(int64_t v) const { return logit_prob(z[v], m, invT, s); }
+  __device__ __forceinline__ void load8(int64_t v, int64_t vend, float out[8]) const {
+    if (v + 8 <= vend && ((reinterpret_cast<uintptr_t>(z + v) & 15u) == 0)) {
+      const uint4 w = *reinterpret_cast<const uint4*>(z + v);
+      const uint32_t h[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        out[2 * j] = logit_prob(__ushort_as_half(lo16(h[j])), m, invT, s);
+        out[2 * j + 1] = logit_prob(__ushort_as_half(hi16(h[j])), m, invT, s);
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) out[j] = v + j < vend ? logit_prob(z[v + j], m, invT, s) : 0.0f;
+    }
+  }
 };
+
+// The 8 fp16 values [v, v + 8) of a row as fp32; entries at or past vend are
+// reported invalid through `ok`.
+__device__ __forceinline__ void load8_half(const __half* z, int64_t v, int64_t vend, float out[8],
+                                           bool ok[8]) {
+  if (v + 8 <= vend && ((reinterpret_cast<uintptr_t>(z + v) & 15u) == 0)) {
+    const uint4 w = *reinterpret_cast<const uint4*>(z + v);
+    const uint32_t h[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      out[2 * j] = __half2float(__ushort_as_half(lo16(h[j])));
+      out[2 * j + 1] = __half2float(__ushort_as_half(hi16(h[j])));
+      ok[2 * j] = ok[2 * j + 1] = true;
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      ok[j] = v + j < vend;
+      out[j] = ok[j] ? __half2float(z[v + j]) : 0.0f;
+    }
+  }
+}
 struct LogitSrc {
   const __half* zp;  // [B, K+1, V]
   const __half* zq;  // [K, B, V]
@@ -164,13 +213,68 @@ __device__ __forceinline__ unsigned long long argmax_key(float v, int64_t idx) {
   return ((unsigned long long)__float_as_uint(v) << 32) | (0xffffffffull - (unsigned long long)idx);
 }
 
+// Block-wide reductions over one value per thread (every thread of the
+// block calls them; `blk` holds one slot per warp).  The results reach
+// every thread.
+template <int NT>
+__device__ __forceinline__ unsigned long long block_sum_u64(unsigned long long v, unsigned long long* blk) {
+  v = warp_sum_u64(v);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) blk[threadIdx.x >> 5] = v;
+  __syncthreads();
+  unsigned long long t = 0;
+#pragma unroll
+  for (int w = 0; w < NT / 32; ++w) t += blk[w];
+  return t;
+}
+
+template <int NT>
+__device__ __forceinline__ unsigned long long block_max_u64(unsigned long long v, unsigned long long* blk) {
+  v = warp_max_u64(v);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) blk[threadIdx.x >> 5] = v;
+  __syncthreads();
+  unsigned long long t = 0;
+#pragma unroll
+  for (int w = 0; w < NT / 32; ++w) t = blk[w] > t ? blk[w] : t;
+  return t;
+}
+
+// Exclusive prefix sum in thread order; `total` receives the block total.
+template <int NT>
+__device__ __forceinline__ unsigned long long block_excl_scan_u64(unsigned long long v, unsigned long long* blk,
+                                                                 unsigned long long& total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  unsigned long long incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned long long t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  __syncthreads();
+  if (lane == 31) blk[warp] = incl;
+  __syncthreads();
+  unsigned long long base = 0, tot = 0;
+#pragma unroll
+  for (int w = 0; w < NT / 32; ++w) {
+    if (w < warp) base += blk[w];
+    tot += blk[w];
+  }
+  total = tot;
+  return base + incl - v;
+}
+
 constexpr int kAcceptThreads = 256;
+static_assert(kAcceptChunk == 8 * kAcceptThreads, "a thread owns 8 consecutive entries of a chunk");
+static_assert(kSoftmaxChunk == 8 * kAcceptThreads, "a thread owns 8 consecutive entries of a chunk");
 
 template <class Src>
 __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a, Src src) {
   griddep_wait();
   griddep_launch_dependents();
   __shared__ unsigned long long red[kAcceptThreads / 32][17];
+  __shared__ unsigned long long blk[kAcceptThreads / 32];
+  __shared__ unsigned long long s_best[17];
   __shared__ int s_n, s_valid, s_last;
   __shared__ unsigned long long s_T;
   __shared__ int s_chunk, s_use_p, s_token;
@@ -219,14 +323,20 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a, Sr
     const bool use_q = n < K;
     const auto qn = src.qrow(b, use_q ? n : 0);
     unsigned long long sr = 0, sp = 0;
-    for (int64_t v = v0 + tid; v < v1; v += kAcceptThreads) {
-      const float pv = pn(v);
-      if (use_q) {
-        const float d = pv - qn(v);
-        sr += fix44(d > 0.0f ? d : 0.0f);
-        sp += fix44(pv);
-      } else {
-        sr += fix44(pv);
+    // thread t: the 8 entries [v0 + 8t, v0 + 8t + 8) of the chunk
+    for (int64_t vb = v0 + 8 * (int64_t)tid; vb < v1; vb += 8 * kAcceptThreads) {
+      float pv[8], qv[8];
+      pn.load8(vb, v1, pv);
+      if (use_q) qn.load8(vb, v1, qv);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (use_q) {
+          const float d = pv[j] - qv[j];
+          sr += fix44(d > 0.0f ? d : 0.0f);
+          sp += fix44(pv[j]);
+        } else {
+          sr += fix44(pv[j]);
+        }
       }
     }
     sr = warp_sum_u64(sr);
@@ -250,9 +360,15 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a, Sr
     for (int i = 0; i <= K; ++i) {
       const auto pi = src.prow(b, i);
       unsigned long long best = 0;
-      for (int64_t v = v0 + tid; v < v1; v += kAcceptThreads) {
-        const unsigned long long k = argmax_key(pi(v), v);
-        best = k > best ? k : best;
+      for (int64_t vb = v0 + 8 * (int64_t)tid; vb < v1; vb += 8 * kAcceptThreads) {
+        float pv[8];
+        pi.load8(vb, v1, pv);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (vb + j >= v1) break;
+          const unsigned long long k = argmax_key(pv[j], vb + j);
+          best = k > best ? k : best;
+        }
       }
       best = warp_max_u64(best);
       if (lane == 0) red[warp][i] = best;
@@ -278,17 +394,24 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a, Sr
   const unsigned long long* pall = a.part + (int64_t)b * a.C * a.slots;
   int32_t* tok = a.tok_out + (int64_t)b * (K + 1);
 
+  // every thread takes the partials of chunks 2t and 2t + 1 (C <= 512)
+  const int c0 = 2 * tid, c1 = 2 * tid + 1;
+  auto partial = [&](int cc, int slot) -> unsigned long long {
+    return cc < a.C ? __ldcg(pall + (int64_t)cc * a.slots + slot) : 0ull;
+  };
+
   if (a.mode == SQ_ACCEPT_GREEDY) {
+    for (int i = 0; i <= K; ++i) {
+      const unsigned long long k0 = partial(c0, i), k1 = partial(c1, i);
+      const unsigned long long best = block_max_u64<kAcceptThreads>(k0 > k1 ? k0 : k1, blk);
+      if (tid == 0) s_best[i] = best;
+    }
+    __syncthreads();
     if (tid == 0) {
       int nn = K;
       int64_t am_n = -1;
       for (int i = 0; i <= K; ++i) {
-        unsigned long long best = 0;
-        for (int cc = 0; cc < a.C; ++cc) {
-          const unsigned long long k = __ldcg(pall + (int64_t)cc * a.slots + i);
-          best = k > best ? k : best;
-        }
-        const int64_t am = (int64_t)(0xffffffffull - (best & 0xffffffffull));
+        const int64_t am = (int64_t)(0xffffffffull - (s_best[i] & 0xffffffffull));
         if (i < nn && i < K && am != xb[i]) nn = i;
         if (i == nn) {
           am_n = am;
@@ -303,34 +426,39 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a, Sr
     return;
   }
 
-  // sampling: pick the row, the total mass, the target and its chunk
+  // sampling: the row's total mass, the target T and the chunk holding it
+  // (block-wide sum, then an exclusive scan of the chunk masses)
+  const unsigned long long r0 = partial(c0, 0), r1 = partial(c1, 0);
+  unsigned long long S = block_sum_u64<kAcceptThreads>(r0 + r1, blk);
+  const int use_p = (S == 0 && n < K) ? 1 : 0;  // block-uniform
+  unsigned long long m0 = r0, m1 = r1;
+  if (use_p) {
+    m0 = partial(c0, 1);
+    m1 = partial(c1, 1);
+    S = block_sum_u64<kAcceptThreads>(m0 + m1, blk);
+  }
+  const int ok = s_valid && S != 0;
+  const unsigned long long T = ok ? scale_floor(ub[K], S) : 0ull;
   if (tid == 0) {
-    unsigned long long S = 0;
-    for (int cc = 0; cc < a.C; ++cc) S += __ldcg(pall + (int64_t)cc * a.slots + 0);
-    int use_p = 0;
-    if (S == 0 && n < K) {
-      for (int cc = 0; cc < a.C; ++cc) S += __ldcg(pall + (int64_t)cc * a.slots + 1);
-      use_p = 1;
-    }
-    int ok = s_valid && S != 0;
     if (s_valid && S == 0) atomicOr(&g_accept_status, SQ_DEV_NO_MASS);
-    const unsigned long long T = ok ? scale_floor(ub[K], S) : 0ull;
-    unsigned long long before = 0;
-    int cs = a.C - 1;
-    for (int cc = 0; cc < a.C; ++cc) {
-      const unsigned long long pc = __ldcg(pall + (int64_t)cc * a.slots + use_p);
-      if (before + pc > T) {
-        cs = cc;
-        break;
-      }
-      before += pc;
-    }
-    s_T = T - before;
-    s_chunk = cs;
+    s_chunk = a.C - 1;
+    s_T = 0;
     s_use_p = use_p;
-    s_valid = ok;
     s_token = -1;
   }
+  unsigned long long total;
+  const unsigned long long excl = block_excl_scan_u64<kAcceptThreads>(m0 + m1, blk, total);
+  if (ok && excl <= T && T < excl + m0 + m1) {  // exactly one thread
+    if (T < excl + m0) {
+      s_chunk = c0;
+      s_T = T - excl;
+    } else {
+      s_chunk = c1;
+      s_T = T - excl - m0;
+    }
+  }
+  __syncthreads();
+  if (tid == 0) s_valid = ok;
   __syncthreads();
   if (s_valid) {
     const auto pn = src.prow(b, n);
@@ -339,39 +467,49 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(AcceptArgs a, Sr
     const int64_t w0 = (int64_t)s_chunk * a.chunk;
     const int64_t w1 = w0 + a.chunk < V ? w0 + a.chunk : V;
     const unsigned long long T = s_T;
-    unsigned long long run = 0;  // mass of the sub-blocks already scanned
-    for (int64_t base = w0; base < w1; base += kAcceptThreads) {
-      const int64_t v = base + tid;
-      unsigned long long R = 0;
-      if (v < w1) {
-        const float pv = pn(v);
+    // thread t holds the 8 entries [w0 + 8t, w0 + 8t + 8) (the chunk is
+    // 8 x the block): local prefix sums, then one block-wide exclusive scan
+    // of the thread totals; the thread whose range holds T finds the token
+    const int64_t vb = w0 + 8 * (int64_t)tid;
+    unsigned long long R[8];
+    {
+      float pv[8], qv[8];
+      pn.load8(vb, w1, pv);
+      if (use_q) qn.load8(vb, w1, qv);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
         if (use_q) {
-          const float d = pv - qn(v);
-          R = fix44(d > 0.0f ? d : 0.0f);
+          const float d = pv[j] - qv[j];
+          R[j] = fix44(d > 0.0f ? d : 0.0f);
         } else {
-          R = fix44(pv);
+          R[j] = fix44(pv[j]);
         }
       }
-      // inclusive block scan of R
-      unsigned long long incl = R;
+    }
+    unsigned long long tot = 0;
 #pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const unsigned long long t = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += t;
+    for (int j = 0; j < 8; ++j) tot += R[j];
+    unsigned long long incl = tot;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const unsigned long long t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
+    }
+    if (lane == 31) red[warp][0] = incl;
+    __syncthreads();
+    unsigned long long wbase = 0;
+    for (int w = 0; w < warp; ++w) wbase += red[w][0];
+    const unsigned long long excl = incl - tot + wbase;
+    if (excl <= T && T < excl + tot) {  // exactly one thread's range holds T
+      unsigned long long c = excl;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        c += R[j];
+        if (c > T) {
+          s_token = (int)(vb + j);
+          break;
+        }
       }
-      if (lane == 31) red[warp][0] = incl;
-      __syncthreads();
-      unsigned long long wbase = 0, total = 0;
-      for (int w = 0; w < kAcceptThreads / 32; ++w) {
-        if (w < warp) wbase += red[w][0];
-        total += red[w][0];
-      }
-      incl += wbase + run;
-      const unsigned long long excl = incl - R;
-      if (excl <= T && incl > T) s_token = (int)v;  // exactly one thread matches
-      __syncthreads();
-      if (s_token >= 0) break;
-      run += total;
     }
   }
   __syncthreads();
@@ -424,10 +562,16 @@ __global__ void __launch_bounds__(kAcceptThreads) softmax_max_kernel(SoftmaxArgs
   const int64_t v1 = v0 + kSoftmaxChunk < a.V ? v0 + kSoftmaxChunk : a.V;
   float mx = -INFINITY;
   int bad = 0;
-  for (int64_t v = v0 + tid; v < v1; v += kAcceptThreads) {
-    const float f = __half2float(z[v]);
-    bad |= !isfinite(f);
-    mx = fmaxf(mx, f);
+  {
+    float f[8];
+    bool ok[8];
+    load8_half(z, v0 + 8 * (int64_t)tid, v1, f, ok);
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if (ok[j]) {
+        bad |= !isfinite(f[j]);
+        mx = fmaxf(mx, f[j]);
+      }
   }
   mx = warp_max(mx);
   bad = __any_sync(0xffffffffu, bad);
@@ -448,20 +592,36 @@ __global__ void __launch_bounds__(kAcceptThreads) softmax_max_kernel(SoftmaxArgs
     s_last = atomicAdd(&a.counter[r], 1u) == (unsigned)(a.C - 1);
   }
   __syncthreads();
-  if (tid == 0 && s_last) {
-    __threadfence();
-    float m = -INFINITY;
-    bool nan = false;
-    for (int cc = 0; cc < a.C; ++cc) {
-      const float pm = __ldcg(a.pmax + r * a.C + cc);
-      nan |= isnan(pm);
-      m = fmaxf(m, pm);
+  if (!s_last) return;
+  __threadfence();
+  // the last CTA of the row: every thread takes chunks t and t + 256
+  float m = -INFINITY;
+  int nan = 0;
+  for (int cc = tid; cc < a.C; cc += kAcceptThreads) {
+    const float pm = __ldcg(a.pmax + r * a.C + cc);
+    nan |= isnan(pm);
+    m = fmaxf(m, pm);
+  }
+  m = warp_max(m);
+  nan = __any_sync(0xffffffffu, nan);
+  __syncthreads();
+  if (lane == 0) {
+    red[warp] = m;
+    red_bad[warp] = nan;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    float mm = -INFINITY;
+    int any_nan = 0;
+    for (int w = 0; w < kAcceptThreads / 32; ++w) {
+      mm = fmaxf(mm, red[w]);
+      any_nan |= red_bad[w];
     }
-    if (nan) {
-      m = __int_as_float(0x7fc00000);
+    if (any_nan) {
+      mm = __int_as_float(0x7fc00000);
       atomicOr(&g_accept_status, SQ_DEV_NONFINITE_LOGIT);
     }
-    a.m[r] = m;
+    a.m[r] = mm;
     a.counter[r] = 0u;
   }
 }
@@ -479,9 +639,14 @@ __global__ void __launch_bounds__(kAcceptThreads) softmax_sum_kernel(SoftmaxArgs
   const int64_t v1 = v0 + kSoftmaxChunk < a.V ? v0 + kSoftmaxChunk : a.V;
   const float m = a.m[r];
   unsigned long long acc = 0;
-  if (isfinite(m))
-    for (int64_t v = v0 + tid; v < v1; v += kAcceptThreads)
-      acc += fixq<40>(exp_neg(__fmul_rn(__fsub_rn(__half2float(z[v]), m), a.invT)));
+  if (isfinite(m)) {
+    float f[8];
+    bool ok[8];
+    load8_half(z, v0 + 8 * (int64_t)tid, v1, f, ok);
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if (ok[j]) acc += fixq<40>(exp_neg(__fmul_rn(__fsub_rn(f[j], m), a.invT)));
+  }
   acc = warp_sum_u64(acc);
   if (lane == 0) red[warp] = acc;
   __syncthreads();
@@ -493,10 +658,12 @@ __global__ void __launch_bounds__(kAcceptThreads) softmax_sum_kernel(SoftmaxArgs
     s_last = atomicAdd(&a.counter[r], 1u) == (unsigned)(a.C - 1);
   }
   __syncthreads();
-  if (tid == 0 && s_last) {
-    __threadfence();
-    unsigned long long S = 0;
-    for (int cc = 0; cc < a.C; ++cc) S += __ldcg(a.psum + r * a.C + cc);
+  if (!s_last) return;
+  __threadfence();
+  unsigned long long part = 0;
+  for (int cc = tid; cc < a.C; cc += kAcceptThreads) part += __ldcg(a.psum + r * a.C + cc);
+  const unsigned long long S = block_sum_u64<kAcceptThreads>(part, red);
+  if (tid == 0) {
     a.s[r] = isfinite(m) ? __double2float_rn(__ull2double_rn(S) * 0x1p-40)
                          : __int_as_float(0x7fc00000);
     a.counter[r] = 0u;
@@ -554,8 +721,15 @@ __global__ void __launch_bounds__(kAcceptThreads) softmax_write_kernel(SoftmaxAr
   const float m = a.m[r], sc = a.s[r];
   const bool ok = isfinite(m) && isfinite(sc);
   float* pr = p + r * a.V;
-  for (int64_t v = v0 + threadIdx.x; v < v1; v += kAcceptThreads)
-    pr[v] = ok ? logit_prob(z[v], m, a.invT, sc) : __int_as_float(0x7fc00000);
+  const int64_t vb = v0 + 8 * (int64_t)threadIdx.x;
+  float f[8];
+  bool in[8];
+  load8_half(z, vb, v1, f, in);
+#pragma unroll
+  for (int j = 0; j < 8; ++j)
+    if (in[j])
+      pr[vb + j] = ok ? __fdiv_rn(exp_neg(__fmul_rn(__fsub_rn(f[j], m), a.invT)), sc)
+                      : __int_as_float(0x7fc00000);
 }
 
 cudaError_t launch_softmax(const SoftmaxArgs& sa, float* p, cudaStream_t st) {

@@ -108,7 +108,7 @@ cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t st);
 
 // Softmax statistics of the logit rows of one accept-from-logits call:
 // target rows zp [rp = B (K+1), V], then draft rows zq [K B, V].
-constexpr int kSoftmaxChunk = 8192;
+constexpr int kSoftmaxChunk = 2048;
 struct SoftmaxArgs {
   const __half* zp;
   const __half* zq;
