@@ -184,6 +184,19 @@ def source_digest(paths):
     return h.hexdigest()[:16]
 
 
+# Sources that build and configure each engine's kernels (template, the
+# format's instantiation unit, device helpers, shared declarations, the
+# planner that picks the configuration).
+_CSRC = os.path.join(ROOT, "paper_2609_21704_gb300", "csrc")
+_COMMON = ("sq_device.cuh", "sq_internal.h", "sq_plan.cu")
+
+
+def kernel_digest(kernel_tag: str) -> str:
+    engine, fmt = kernel_tag.split("_")[:2]
+    files = (("sq_gemv.cuh", f"sq_gemv_{fmt}.cu") if engine == "gemv" else ("sq_tc.cu",)) + _COMMON
+    return source_digest([os.path.join(_CSRC, f) for f in files])
+
+
 def profiled_traffic(kernel_tag: str, digest: str):
     """DRAM bytes per launch of `kernel_tag` from a committed ncu summary,
     or None when the kernel source changed since the capture."""
@@ -453,8 +466,7 @@ def main():
     gu_bytes = gu_projs[0].weight_bytes(args.draft) + 2 * B * (shape.hidden + shape.intermediate)
     gu16_bytes = gu_projs[0].weight_bytes("fp16") + 2 * Mv * (shape.hidden + shape.intermediate)
     achieved = gu_bytes / t_gu / 1e9
-    digest = source_digest(glob.glob(os.path.join(ROOT, "paper_2609_21704_gb300", "csrc", "*")))
-    traffic = profiled_traffic(kernel_tag, digest)
+    traffic = profiled_traffic(kernel_tag, kernel_digest(kernel_tag))
 
     # ---- end to end through the public API with host buffers
     e2e = None

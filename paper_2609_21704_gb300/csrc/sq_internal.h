@@ -11,8 +11,14 @@ namespace sq {
 
 constexpr int kNumSMs = 152;  // GB300: 2 dies x 76 SMs (queried at run time too)
 
+// sq_plan.cu: device properties and the choice of engine and configuration
 int device_sm_count();
-bool pdl_enabled();  // SQ_PDL environment knob, read once
+int device_max_smem();  // opt-in shared memory per block
+bool pdl_enabled();     // SQ_PDL environment knob, read once
+int64_t weights_per_piece(int wkind);         // weights in one 16-byte piece of a row
+int64_t row_bytes_of(int wkind, int64_t K);   // bytes of one weight row
+int gemv_cap_mr(int wkind, int64_t K);        // largest activation-row chunk whose x fits
+bool use_tensor_cores(int wkind, int M, int64_t N, int64_t K, int epi);
 
 // Launch with programmatic dependent launch allowed: the kernel may begin
 // while the previous kernel on the stream drains; it must call
