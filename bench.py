@@ -417,11 +417,20 @@ def main():
                                                      n_out, tok_out, ws_l, stream))
         g_smpl = capture(lambda: sq.sq_sample_logits(zq[0], u_draft[0], temperature, samp[0], ws_s,
                                                      stream))
+
+        # direct decoding with the FP16 parent (the paper's path for high-
+        # complexity prompts, and the baseline its speedups are quoted
+        # against): one pass at M = B and a sample per token
+        def direct_token():
+            stk.run_pass(stack, "fp16", bd, stream, logits=zq[0])
+            sq.sq_sample_logits(zq[0], u_draft[0], temperature, samp[0], ws_s, stream)
+        g_direct = capture(direct_token)
         t_draft = timed(g_draft, reps) / reps
         t_ver = timed(g_ver, reps) / reps
         t_acc = timed(g_acc, reps) / reps
         t_accl = timed(g_accl, reps) / reps
         t_smpl = timed(g_smpl, reps) / reps
+        t_direct = timed(g_direct, reps) / reps
         # the same passes as separate sq_linear_ex calls
         g_draft_u = capture(lambda: stk.run_pass_unchained(stack, args.draft, bd, stream))
         g_ver_u = capture(lambda: stk.run_pass_unchained(stack, "fp16", bv, stream))
@@ -553,6 +562,9 @@ def main():
             "fp16_gateup_silu_m%d_us" % Mv: 1e6 * t_gu16,
             "fp16_gateup_silu_gbs": gu16_bytes / t_gu16 / 1e9,
             "launches_per_pass": stack.launches_per_pass(),
+            "direct_fp16_ms_per_token": 1e3 * t_direct,
+            "direct_fp16_tokens_per_s": B * world / t_direct,
+            "speedup_vs_direct_fp16": value / (B * world / t_direct),
             "prefill_m256_fp16_ms": 1e3 * t_pf16,
             "prefill_m256_fp16_tflops": pf_flops / t_pf16 / 1e12,
             "prefill_m256_%s_ms" % args.draft: 1e3 * t_pfd,

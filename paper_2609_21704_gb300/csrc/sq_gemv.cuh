@@ -104,8 +104,19 @@ struct Unroll {
 // own R rows with LPR lanes; LPR is chosen so that a row's 16-byte pieces
 // divide evenly among the lanes (no idle lanes), and the groups of a warp
 // read the same x slots (shared-memory broadcast).
+// Minimum resident CTAs per SM the compiler must allow (register cap).  The
+// single-row INT4 fused gate/up (M = 1) runs at 4 (64 registers): its
+// 4480-tile 1.5B matrix then starts every tile in the first wave (draft
+// pass 485 -> 462 us measured); every other configuration keeps the
+// registers it needs.
+template <int WK, int MR, int R, bool SILU>
+struct GemvMinBlocks {
+  static constexpr int value = (WK == WK_INT4 && MR == 1 && R == 1 && SILU) ? 4 : 1;
+};
+
 template <int WK, int MR, int R, bool SILU, int LPR>
-__global__ void __launch_bounds__(kGemvThreads) gemv_kernel(const GemvArgs a) {
+__global__ void __launch_bounds__(kGemvThreads, (GemvMinBlocks<WK, MR, R, SILU>::value))
+    gemv_kernel(const GemvArgs a) {
   using T = WTraits<WK>;
   constexpr int SUB = T::kSub;
   constexpr int WR = SILU ? 2 * R : R;  // weight rows per lane group
