@@ -93,6 +93,22 @@ __device__ __forceinline__ void int4x8_to_f16x2(uint32_t w, uint32_t out[4]) {
   asm("fma.rn.f16x2 %0, %1, %2, %3;" : "=r"(out[3]) : "r"(d), "r"(SIXTEENTH), "r"(SUB_HI));
 }
 
+// The same eight codes as the raw fp16 values OR-ed onto 1024 (no bias
+// removal): out[0] = (1024 + n0, 1024 + n4), out[1] = (1024 + 16 n1,
+// 1024 + 16 n5), out[2] = (1024 + n2, 1024 + n6), out[3] = (1024 + 16 n3,
+// 1024 + 16 n7), n_j = c_j + 8 the stored nibble.  Even k carry 1024 + n,
+// odd k 1024 + 16 n; the linear kernel removes the offsets per 32-weight
+// piece with precomputed activation sums.
+__device__ __forceinline__ void int4x8_to_magic(uint32_t w, uint32_t out[4]) {
+  const uint32_t MAGIC = 0x64006400u;
+  const uint32_t LO = 0x000f000fu, HI = 0x00f000f0u;
+  const uint32_t w8 = w >> 8;
+  asm("lop3.b32 %0, %1, %2, %3, 0xea;" : "=r"(out[0]) : "r"(w), "r"(LO), "r"(MAGIC));
+  asm("lop3.b32 %0, %1, %2, %3, 0xea;" : "=r"(out[1]) : "r"(w), "r"(HI), "r"(MAGIC));
+  asm("lop3.b32 %0, %1, %2, %3, 0xea;" : "=r"(out[2]) : "r"(w8), "r"(LO), "r"(MAGIC));
+  asm("lop3.b32 %0, %1, %2, %3, 0xea;" : "=r"(out[3]) : "r"(w8), "r"(HI), "r"(MAGIC));
+}
+
 // ---- packed fp32 pairs (f32x2) ------------------------------------------
 // Accumulators and operands of fma.rn.f32x2 live in 64-bit registers holding
 // (low = first, high = second) fp32 values.

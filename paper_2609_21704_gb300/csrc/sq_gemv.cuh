@@ -76,6 +76,22 @@ __device__ __forceinline__ float dot8_int4order(const uint32_t c[4], const uint4
   return acc;
 }
 
+// INT4 with the offsets left in (int4x8_to_magic): the even-k products
+// (1024 + n) x go to `even`, the odd-k products (1024 + 16 n) x to `odd`,
+// both exact in fp32.  For a piece, sum_k c_k x_k = even + odd / 16 -
+// (1032 X_even + 72 X_odd), X the piece's activation sums.
+__device__ __forceinline__ void dot8_int4magic(const uint32_t v[4], const uint4 xq, float& even,
+                                               float& odd) {
+  even = fma_h(lo16(v[0]), lo16(xq.x), even);  // k0
+  odd = fma_h(lo16(v[1]), hi16(xq.x), odd);    // k1
+  even = fma_h(lo16(v[2]), lo16(xq.y), even);  // k2
+  odd = fma_h(lo16(v[3]), hi16(xq.y), odd);    // k3
+  even = fma_h(hi16(v[0]), lo16(xq.z), even);  // k4
+  odd = fma_h(hi16(v[1]), hi16(xq.z), odd);    // k5
+  even = fma_h(hi16(v[2]), lo16(xq.w), even);  // k6
+  odd = fma_h(hi16(v[3]), hi16(xq.w), odd);    // k7
+}
+
 // Same for weights already in natural order: pairs (w0,w1),(w2,w3),...
 __device__ __forceinline__ float dot8_natural(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3,
                                               const uint4 xq, float acc) {
@@ -211,6 +227,28 @@ __global__ void __launch_bounds__(kGemvThreads, (GemvMinBlocks<WK, MR, R, SILU>:
       if (base + b * kGemvThreads < total) xs[base + b * kGemvThreads] = v[b];
   }
   __syncthreads();
+  // INT4: per (row m, piece p) the offset 1032 X_even + 72 X_odd that the
+  // magic-valued products carry (X = the piece's 32 activations summed over
+  // even / odd k), behind x in shared memory
+  float* xoff = reinterpret_cast<float*>(xs + total);
+  if constexpr (WK == WK_INT4) {
+    for (int idx = threadIdx.x; idx < MR * a.ppad; idx += kGemvThreads) {
+      const int m = idx / a.ppad, pp = idx - m * a.ppad;
+      float xe = 0.0f, xo = 0.0f;
+#pragma unroll
+      for (int i = 0; i < SUB; ++i) {
+        const uint4 q = xs[m * chunks_per_m + ((pp >> 5) * SUB + i) * 32 + (pp & 31)];
+        const uint32_t h[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          xe += __half2float(__ushort_as_half(lo16(h[j])));
+          xo += __half2float(__ushort_as_half(hi16(h[j])));
+        }
+      }
+      xoff[idx] = fmaf(1032.0f, xe, 72.0f * xo);
+    }
+    __syncthreads();
+  }
 
   for (int64_t tile = gwarp; tile < t_end; tile += nwarps) {
     prefetch_tile(tile + (int64_t)(kPrefetchTiles + 1) * nwarps);
@@ -229,11 +267,11 @@ __global__ void __launch_bounds__(kGemvThreads, (GemvMinBlocks<WK, MR, R, SILU>:
         const int p = j * LPR + ll;      // this lane's piece of the row
         const int xsl = ((p >> 5) * SUB) * 32 + (p & 31);  // x slot of sub-chunk 0
         if constexpr (WK == WK_INT4) {
-          float part[WR][MR];
+          float pe[WR][MR], po[WR][MR];
 #pragma unroll
           for (int r = 0; r < WR; ++r)
 #pragma unroll
-            for (int m = 0; m < MR; ++m) part[r][m] = 0.0f;
+            for (int m = 0; m < MR; ++m) pe[r][m] = po[r][m] = 0.0f;
 #pragma unroll
           for (int i = 0; i < SUB; ++i) {
             uint32_t c[WR][4];
@@ -241,19 +279,22 @@ __global__ void __launch_bounds__(kGemvThreads, (GemvMinBlocks<WK, MR, R, SILU>:
             for (int r = 0; r < WR; ++r) {
               const uint4 w = wv[u][r];
               const uint32_t word = i == 0 ? w.x : i == 1 ? w.y : i == 2 ? w.z : w.w;
-              int4x8_to_f16x2(word, c[r]);
+              int4x8_to_magic(word, c[r]);
             }
 #pragma unroll
             for (int m = 0; m < MR; ++m) {
               const uint4 xq = xs[m * chunks_per_m + xsl + i * 32];
 #pragma unroll
-              for (int r = 0; r < WR; ++r) part[r][m] = dot8_int4order(c[r], xq, part[r][m]);
+              for (int r = 0; r < WR; ++r) dot8_int4magic(c[r], xq, pe[r][m], po[r][m]);
             }
           }
 #pragma unroll
-          for (int r = 0; r < WR; ++r)
+          for (int m = 0; m < MR; ++m) {
+            const float off = xoff[m * a.ppad + p];  // 1032 X_even + 72 X_odd of this piece
 #pragma unroll
-            for (int m = 0; m < MR; ++m) acc[r][m] = fmaf(sv[u][r], part[r][m], acc[r][m]);
+            for (int r = 0; r < WR; ++r)
+              acc[r][m] = fmaf(sv[u][r], fmaf(po[r][m], 0.0625f, pe[r][m]) - off, acc[r][m]);
+          }
         } else if constexpr (WK == WK_FP8) {
 #pragma unroll
           for (int i = 0; i < SUB; ++i) {

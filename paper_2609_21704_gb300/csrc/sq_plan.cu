@@ -55,7 +55,8 @@ int64_t row_bytes_of(int wk, int64_t K) {
 size_t gemv_smem_bytes(int wk, int mr, int64_t K) {
   const int64_t pieces = K / weights_per_piece(wk);
   const int64_t ppad = (pieces + 31) / 32 * 32;
-  return (size_t)mr * (size_t)ppad * (size_t)sub_of(wk) * 16u;
+  // staged x, plus one fp32 offset per (row, piece) for INT4
+  return (size_t)mr * (size_t)ppad * ((size_t)sub_of(wk) * 16u + (wk == SQ_W_INT4 ? 4u : 0u));
 }
 
 // Compiled activation-row counts (sq_gemv.cuh instantiations).
