@@ -97,6 +97,9 @@ def _load():
         "oq_sample": (ctypes.c_int, [P, P, I64, I64, P]),
         "oq_enum_sweep": (ctypes.c_int, [P, P, P, P, I64, I64, ctypes.c_int, ctypes.c_int,
                                          ctypes.c_int, P]),
+        "oq_rmsnorm": (None, [P, P, I64, I64, ctypes.c_double, P]),
+        "oq_rope": (None, [P, P, I64, I64, I64, ctypes.c_double]),
+        "oq_attention": (None, [P, P, P, P, I64, I64, I64, I64, I64, P]),
         "oq_exp_neg": (ctypes.c_float, [ctypes.c_float]),
         "oq_exp_neg_array": (None, [P, I64, P]),
         "oq_softmax_row": (ctypes.c_int, [P, I64, ctypes.c_float, P]),
@@ -326,3 +329,37 @@ def sample_logits(z, u, T: float = 1.0):
     if st == BAD_ARG:
         raise ValueError("oq_sample_logits: bad arguments")
     return st, t
+
+
+# ---- the decoder around the linear stack ----------------------------------------
+
+def rmsnorm(x, gamma, eps: float = 1e-6) -> np.ndarray:
+    """y = x / sqrt(mean(x^2) + eps) * gamma in fp64; x [M, H], gamma [H]."""
+    xa = _c(np.atleast_2d(x), np.float64)
+    ga = _c(gamma, np.float64)
+    M, H = xa.shape
+    y = np.empty_like(xa)
+    _load().oq_rmsnorm(_ptr(xa), _ptr(ga), M, H, float(eps), _ptr(y))
+    return y
+
+
+def rope(x, pos, nheads: int, head_dim: int, theta: float = 1e6) -> np.ndarray:
+    """Rotary embedding (rotate-half pairs d, d + D/2) of rows x [M, nheads*D]."""
+    xa = _c(np.atleast_2d(x), np.float64).copy()
+    pa = _c(pos, np.int64)
+    M = xa.shape[0]
+    _load().oq_rope(_ptr(xa), _ptr(pa), M, nheads, head_dim, float(theta))
+    return xa
+
+
+def attention(q, k, v, qpos) -> np.ndarray:
+    """q [T, Hq, D], k/v [L, Hkv, D]; query t sees keys 0..qpos[t] -> [T, Hq, D]."""
+    qa = _c(q, np.float64)
+    ka = _c(k, np.float64)
+    va = _c(v, np.float64)
+    T, Hq, D = qa.shape
+    L, Hkv, _ = ka.shape
+    pa = _c(qpos, np.int64)
+    out = np.empty((T, Hq, D), np.float64)
+    _load().oq_attention(_ptr(qa), _ptr(ka), _ptr(va), _ptr(pa), T, L, Hq, Hkv, D, _ptr(out))
+    return out

@@ -465,3 +465,60 @@ int oq_sample_logits(const uint16_t* z, const float* u, int64_t B, int64_t V,
   free(p);
   return st;
 }
+
+/* ---- decoder: RMSNorm, RoPE, attention ----------------------------------- */
+
+void oq_rmsnorm(const double* x, const double* gamma, int64_t M, int64_t H, double eps, double* y) {
+  for (int64_t m = 0; m < M; ++m) {
+    double ss = 0.0;
+    for (int64_t h = 0; h < H; ++h) ss += x[m * H + h] * x[m * H + h];
+    const double r = 1.0 / sqrt(ss / (double)H + eps);
+    for (int64_t h = 0; h < H; ++h) y[m * H + h] = x[m * H + h] * r * gamma[h];
+  }
+}
+
+void oq_rope(double* x, const int64_t* pos, int64_t M, int64_t nheads, int64_t D, double theta) {
+  const int64_t half = D / 2;
+  for (int64_t m = 0; m < M; ++m)
+    for (int64_t h = 0; h < nheads; ++h) {
+      double* r = x + (m * nheads + h) * D;
+      for (int64_t d = 0; d < half; ++d) {
+        const double f = pow(theta, -2.0 * (double)d / (double)D);
+        const double a = (double)pos[m] * f;
+        const double c = cos(a), s = sin(a);
+        const double x1 = r[d], x2 = r[d + half];
+        r[d] = x1 * c - x2 * s;
+        r[d + half] = x2 * c + x1 * s;
+      }
+    }
+}
+
+void oq_attention(const double* q, const double* k, const double* v, const int64_t* qpos,
+                  int64_t T, int64_t L, int64_t Hq, int64_t Hkv, int64_t D, double* out) {
+  const int64_t G = Hq / Hkv;
+  const double scale = 1.0 / sqrt((double)D);
+  double* w = (double*)malloc((size_t)(L > 0 ? L : 1) * sizeof(double));
+  for (int64_t t = 0; t < T; ++t)
+    for (int64_t h = 0; h < Hq; ++h) {
+      const int64_t kh = h / G;
+      const double* qr = q + (t * Hq + h) * D;
+      int64_t n = qpos[t] + 1 < L ? qpos[t] + 1 : L;  /* keys 0 .. qpos[t] */
+      double mx = -INFINITY;
+      for (int64_t j = 0; j < n; ++j) {
+        double dot = 0.0;
+        for (int64_t d = 0; d < D; ++d) dot += qr[d] * k[(j * Hkv + kh) * D + d];
+        w[j] = dot * scale;
+        if (w[j] > mx) mx = w[j];
+      }
+      double sum = 0.0;
+      for (int64_t j = 0; j < n; ++j) {
+        w[j] = exp(w[j] - mx);
+        sum += w[j];
+      }
+      double* o = out + (t * Hq + h) * D;
+      for (int64_t d = 0; d < D; ++d) o[d] = 0.0;
+      for (int64_t j = 0; j < n; ++j)
+        for (int64_t d = 0; d < D; ++d) o[d] += w[j] / sum * v[(j * Hkv + kh) * D + d];
+    }
+  free(w);
+}

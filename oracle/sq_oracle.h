@@ -131,6 +131,27 @@ int oq_accept_logits(const uint16_t* zp, const uint16_t* zq, const int32_t* draf
 int oq_sample_logits(const uint16_t* z, const float* u, int64_t B, int64_t V,
                      float T, int32_t* tokens);
 
+/* ---- the decoder around the linear stack (attention, KV cache) -----------
+ * Sec. III-D.2/3 run the full model; Sec. III-D.4 rolls the parent's state
+ * back to the first rejected token ("recommence ... starting with the first
+ * token that was rejected").  The paper states no model internals; these
+ * follow the Qwen2.5 decoder the workloads are shaped after, in fp64:
+ *   RMSNorm   y = x / sqrt(mean(x^2) + eps) * gamma
+ *   RoPE      for d < D/2, f_d = theta^(-2d/D), a = pos * f_d:
+ *             (x_d, x_{d+D/2}) -> (x_d cos a - x_{d+D/2} sin a,
+ *                                   x_{d+D/2} cos a + x_d sin a)
+ *   attention out_h = softmax_j(q_h . k_j / sqrt(D)) v_j over the cache
+ *             positions j <= pos of the query, key/value head h / (Hq/Hkv)
+ *             (grouped-query attention). */
+/* x, y [M, H] (x values), gamma [H]. */
+void oq_rmsnorm(const double* x, const double* gamma, int64_t M, int64_t H, double eps, double* y);
+/* In place on rows [M, nheads * D] at positions pos[M]. */
+void oq_rope(double* x, const int64_t* pos, int64_t M, int64_t nheads, int64_t D, double theta);
+/* q [T, Hq, D] already rotated, k and v [L, Hkv, D] (k rotated), query t at
+ * position qpos[t] sees keys j <= qpos[t] (j < L) -> out [T, Hq, D]. */
+void oq_attention(const double* q, const double* k, const double* v, const int64_t* qpos,
+                  int64_t T, int64_t L, int64_t Hq, int64_t Hkv, int64_t D, double* out);
+
 /* ---- exhaustive-enumeration harness (sq_enumerate.c) --------------------- */
 /* Runs oq_accept on one sequence 2^grid_bits times, with the uniform at
  * position `pos` set to m * 2^-grid_bits for every m, the others taken from
