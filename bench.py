@@ -445,6 +445,40 @@ def main():
         g_pfd = pass_graph(args.draft, bp)
         t_pfd = timed(g_pfd, reps_pf) / reps_pf
         del g_pf16, g_pfd, bp
+
+        # the decoder step around the stack (RMSNorm, RoPE, KV cache,
+        # grouped-query attention) at a 1000-token context: each pass alone,
+        # a whole speculative cycle on decoder passes (drafts write their
+        # logits slot and sample, verify, accept, cache rollback) and direct
+        # decoding with the FP16 parent
+        ctx = 1000
+        dd = stk.DecoderState(stack, B, 1, ctx + 64, ctx, seed=40 + rank)
+        dv = stk.DecoderState(stack, B, K + 1, ctx + 64, ctx, seed=50 + rank)
+        new_len = torch.empty(B, dtype=torch.int32, device=dev)
+
+        def dec_cycle():
+            for k in range(K):
+                stk.decoder_pass(stack, args.draft, dd, stream, logits=zq[k])
+                sq.sq_sample_logits(zq[k], u_draft[k], temperature, samp[k], ws_s, stream)
+            stk.decoder_pass(stack, "fp16", dv, stream)
+            sq.sq_accept_logits(dv.logits.view(B, K + 1, V), zq, td, tu, temperature,
+                                sq.SQ_ACCEPT_SAMPLE, n_out, tok_out, ws_l, stream)
+            sq.sq_kv_rollback(dv.pos0, n_out, K + 1, new_len, stream)
+
+        def dec_direct():
+            stk.decoder_pass(stack, "fp16", dd, stream, logits=zq[0])
+            sq.sq_sample_logits(zq[0], u_draft[0], temperature, samp[0], ws_s, stream)
+
+        g_dd = capture(lambda: stk.decoder_pass(stack, args.draft, dd, stream))
+        g_dv = capture(lambda: stk.decoder_pass(stack, "fp16", dv, stream))
+        g_dc = capture(dec_cycle)
+        g_ddir = capture(dec_direct)
+        t_dd = timed(g_dd, reps) / reps
+        t_dv = timed(g_dv, reps) / reps
+        reps_c = max(10, reps // 4)
+        t_dc = timed(g_dc, reps_c) / reps_c
+        t_ddir = timed(g_ddir, reps) / reps
+        del g_dd, g_dv, g_dc, g_ddir, dd, dv
     tensor_peak, tensor_peak_kind = measured_tensor_peak()
     pf_flops = 2.0 * 256 * stack.params()
     draft_bytes = stack.weight_bytes(args.draft) + stack.activation_bytes(B)
@@ -565,6 +599,13 @@ def main():
             "direct_fp16_ms_per_token": 1e3 * t_direct,
             "direct_fp16_tokens_per_s": B * world / t_direct,
             "speedup_vs_direct_fp16": value / (B * world / t_direct),
+            "decoder_context": ctx,
+            "decoder_draft_pass_ms": 1e3 * t_dd,
+            "decoder_verify_pass_ms": 1e3 * t_dv,
+            "decoder_cycle_ms": 1e3 * t_dc,
+            "decoder_tokens_per_s": B * world * mean_tokens / t_dc,
+            "decoder_direct_fp16_tokens_per_s": B * world / t_ddir,
+            "decoder_speedup_vs_direct_fp16": (mean_tokens / t_dc) / (1.0 / t_ddir),
             "prefill_m256_fp16_ms": 1e3 * t_pf16,
             "prefill_m256_fp16_tflops": pf_flops / t_pf16 / 1e12,
             "prefill_m256_%s_ms" % args.draft: 1e3 * t_pfd,

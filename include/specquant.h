@@ -75,6 +75,7 @@ typedef enum { SQ_ACCEPT_SAMPLE = 0, SQ_ACCEPT_GREEDY = 1 } sq_accept_mode;
 #define SQ_DEV_BAD_UNIFORM      0x8u  /* resampling uniform not in [0,1)     */
 #define SQ_DEV_TIMEOUT          0x10u /* a kernel gave up a bounded wait     */
 #define SQ_DEV_NONFINITE_LOGIT  0x20u /* a logit row held inf or NaN         */
+#define SQ_DEV_BAD_POSITION     0x40u /* a token position outside the cache  */
 
 /* Thread-local text of the last error raised on this host thread. */
 SQ_API const char* sq_last_error(void);
@@ -285,6 +286,48 @@ SQ_API sq_status sq_sample_logits(const void* z, const float* u, int B, int64_t 
 SQ_API size_t sq_softmax_workspace_bytes(int64_t R, int64_t V);
 SQ_API sq_status sq_softmax(const void* z, int64_t R, int64_t V, float temperature, float* p,
                             void* workspace, size_t ws_bytes, sq_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * The decoder around the linear stack.  Sec. III-D.2/3 run the whole model
+ * for draft and verify; Sec. III-D.4 restarts from the first rejected
+ * token, so each model's KV cache keeps only the accepted prefix.  The
+ * paper gives no model internals; these follow the Qwen2.5 decoder:
+ *
+ * sq_rmsnorm: y[m, :] = x[m, :] / sqrt(mean(x[m, :]^2) + eps) * gamma, fp32
+ *   arithmetic, fp16 x, gamma [H], y [M, H] (y may equal x).
+ *
+ * Attention layout: qkv fp16 [B*T, (Hq + 2 Hkv) * D], the fused q/k/v
+ * projection's output for T new tokens of each of B sequences (row b*T + t:
+ * q heads, then k heads, then v heads); D = 128; Hq a multiple of Hkv; token
+ * t of sequence b is at position pos0[b] + t (pos0 int32 [B], device).
+ * Caches k_cache, v_cache fp16 [B, Hkv, max_ctx, D].  RoPE rotates pairs
+ * (d, d + D/2) by pos * theta^(-2d/D) (angle computed in fp64).
+ *
+ * sq_kv_append: rotates the new keys and writes keys and values into the
+ *   caches at their positions.  A position outside [0, max_ctx) writes
+ *   nothing and sets SQ_DEV_BAD_POSITION.
+ * sq_attention: out fp16 [B*T, Hq * D]: for query head h of token t,
+ *   softmax_j(q . k_j / sqrt(D)) v_j over cache positions j <= pos0[b] + t
+ *   of key/value head h / (Hq / Hkv), q rotated at its position; the keys
+ *   of the current tokens must already be appended.  Accumulation in fp32.
+ *   T <= 32, (Hq / Hkv) * T <= 200, max_ctx <= 2^17.  workspace: sq_attention_workspace_bytes(...)
+ *   bytes, 16-byte aligned (no zero-fill needed).
+ * sq_kv_rollback: len[b] = base[b] + min(n_accepted[b] + 1, limit), or
+ *   base[b] when n_accepted[b] < 0 (the cache length to keep after
+ *   acceptance: the verified prefix plus the accepted drafts); int32
+ *   device arrays. */
+SQ_API sq_status sq_rmsnorm(const void* x, const void* gamma, int M, int64_t H, float eps, void* y,
+                            sq_stream_t stream);
+SQ_API sq_status sq_kv_append(const void* qkv, int B, int T, int Hq, int Hkv, int D,
+                              const int32_t* pos0, float theta, void* k_cache, void* v_cache,
+                              int64_t max_ctx, sq_stream_t stream);
+SQ_API size_t sq_attention_workspace_bytes(int B, int T, int Hq, int Hkv, int D, int64_t max_ctx);
+SQ_API sq_status sq_attention(const void* qkv, int B, int T, int Hq, int Hkv, int D,
+                              const int32_t* pos0, float theta, const void* k_cache,
+                              const void* v_cache, int64_t max_ctx, void* out, void* workspace,
+                              size_t ws_bytes, sq_stream_t stream);
+SQ_API sq_status sq_kv_rollback(const int32_t* base, const int32_t* n_accepted, int B, int limit,
+                                int32_t* len, sq_stream_t stream);
 
 /* ------------------------------------------------------------------------
  * sq_accept_noalloc: sq_accept without a caller workspace.  The paper has

@@ -28,7 +28,8 @@ __all__ = [
     "sq_linear_ex", "sq_accept_workspace_bytes", "sq_accept", "sq_sample", "sq_check",
     "sq_version", "sq_accept_noalloc", "sq_linear_path", "sq_linear_chain", "SqLinearOp",
     "sq_accept_logits_workspace_bytes", "sq_accept_logits", "sq_sample_logits",
-    "sq_softmax_workspace_bytes", "sq_softmax",
+    "sq_softmax_workspace_bytes", "sq_softmax", "sq_rmsnorm", "sq_kv_append",
+    "sq_attention_workspace_bytes", "sq_attention", "sq_kv_rollback",
     "EXPORTED_SYMBOLS",
 ]
 
@@ -38,7 +39,7 @@ SQ_ACCEPT_SAMPLE, SQ_ACCEPT_GREEDY = 0, 1
 SQ_EPI_NONE, SQ_EPI_SILU_GATE, SQ_EPI_RESIDUAL = 0, 1, 2
 SQ_W_FP16, SQ_W_INT4, SQ_W_FP8 = 0, 1, 2
 SQ_DEV_NONFINITE_WEIGHT, SQ_DEV_BAD_DRAFT_TOKEN, SQ_DEV_NO_MASS, SQ_DEV_BAD_UNIFORM = 1, 2, 4, 8
-SQ_DEV_TIMEOUT, SQ_DEV_NONFINITE_LOGIT = 0x10, 0x20
+SQ_DEV_TIMEOUT, SQ_DEV_NONFINITE_LOGIT, SQ_DEV_BAD_POSITION = 0x10, 0x20, 0x40
 
 _P = ctypes.c_void_p
 _I64 = ctypes.c_int64
@@ -67,6 +68,12 @@ _SIGS = {
     "sq_sample_logits": (_INT, [_P, _P, _INT, _I64, ctypes.c_float, _P, _P, _SIZE, _P]),
     "sq_softmax_workspace_bytes": (_SIZE, [_I64, _I64]),
     "sq_softmax": (_INT, [_P, _I64, _I64, ctypes.c_float, _P, _P, _SIZE, _P]),
+    "sq_rmsnorm": (_INT, [_P, _P, _INT, _I64, ctypes.c_float, _P, _P]),
+    "sq_kv_append": (_INT, [_P, _INT, _INT, _INT, _INT, _INT, _P, ctypes.c_float, _P, _P, _I64, _P]),
+    "sq_attention_workspace_bytes": (_SIZE, [_INT, _INT, _INT, _INT, _INT, _I64]),
+    "sq_attention": (_INT, [_P, _INT, _INT, _INT, _INT, _INT, _P, ctypes.c_float, _P, _P, _I64, _P, _P,
+                            _SIZE, _P]),
+    "sq_kv_rollback": (_INT, [_P, _P, _INT, _INT, _P, _P]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGS)
 
@@ -225,6 +232,37 @@ def sq_softmax(z, temperature, p, workspace, stream=None) -> None:
     _check("sq_softmax", load().sq_softmax(_ptr(z), R, V, float(temperature), _ptr(p), _ptr(workspace),
                                            workspace.numel() * workspace.element_size(),
                                            _stream(stream)))
+
+
+def sq_rmsnorm(x, gamma, eps, y, stream=None) -> None:
+    M, H = x.shape
+    _check("sq_rmsnorm", load().sq_rmsnorm(_ptr(x), _ptr(gamma), M, H, float(eps), _ptr(y),
+                                           _stream(stream)))
+
+
+def sq_kv_append(qkv, B, T, Hq, Hkv, pos0, theta, k_cache, v_cache, stream=None) -> None:
+    """qkv fp16 [B*T, (Hq+2Hkv)*128]; caches fp16 [B, Hkv, max_ctx, 128]."""
+    _check("sq_kv_append", load().sq_kv_append(_ptr(qkv), B, T, Hq, Hkv, 128, _ptr(pos0), float(theta),
+                                               _ptr(k_cache), _ptr(v_cache), k_cache.shape[2],
+                                               _stream(stream)))
+
+
+def sq_attention_workspace_bytes(B, T, Hq, Hkv, max_ctx) -> int:
+    return int(load().sq_attention_workspace_bytes(B, T, Hq, Hkv, 128, max_ctx))
+
+
+def sq_attention(qkv, B, T, Hq, Hkv, pos0, theta, k_cache, v_cache, out, workspace,
+                 stream=None) -> None:
+    """out fp16 [B*T, Hq*128] = causal GQA attention of the new tokens over the caches."""
+    _check("sq_attention", load().sq_attention(
+        _ptr(qkv), B, T, Hq, Hkv, 128, _ptr(pos0), float(theta), _ptr(k_cache), _ptr(v_cache),
+        k_cache.shape[2], _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
+        _stream(stream)))
+
+
+def sq_kv_rollback(base, n_accepted, limit, length, stream=None) -> None:
+    _check("sq_kv_rollback", load().sq_kv_rollback(_ptr(base), _ptr(n_accepted), base.numel(), limit,
+                                                   _ptr(length), _stream(stream)))
 
 
 def sq_accept_workspace_bytes(B: int, K: int, V: int) -> int:

@@ -1,0 +1,384 @@
+// sq_attention.cu -- the decoder around the linear stack: RMSNorm, rotary
+// embedding with the KV-cache append, grouped-query decode attention over
+// the cache, and the rollback of cache lengths after acceptance.
+//
+// Sec. III-D.2/3 run the whole model for the draft and verify passes;
+// Sec. III-D.4 restarts from the first rejected token, so each model's
+// cache keeps only the accepted prefix.  Definitions (no model internals
+// are given in the paper; these are the Qwen2.5 decoder's):
+//   RMSNorm   y = x / sqrt(mean(x^2) + eps) * gamma       (fp32, fp16 out)
+//   RoPE      pairs (d, d + D/2), angle pos * theta^(-2d/D) (fp64 angle)
+//   attention softmax(q . k / sqrt(D)) v over cache positions <= the
+//             query's position; query head h reads key/value head
+//             h / (Hq / Hkv).
+// Layouts: qkv rows [B*T, (Hq + 2 Hkv) D] (q heads, k heads, v heads, the
+// fused projection's output); caches [B, Hkv, max_ctx, D] fp16; attention
+// output rows [B*T, Hq D].  Token t of sequence b sits at position
+// pos0[b] + t.
+//
+// Attention is split over 64-key chunks of the cache (one CTA per
+// (sequence, key/value head, chunk)): all G * T queries of the group read
+// the chunk once from shared memory, then a combine kernel merges the
+// chunks' (max, sum, weighted value) partials.  Bound: the cache bytes
+// (2 * pos * Hkv * D * 2 per sequence) and, for long query groups, CUDA-core
+// arithmetic (G * T * 2 D flops per cached key).
+#include <math.h>
+
+#include "sq_internal.h"
+
+namespace sq {
+
+__device__ unsigned int g_attn_status;
+
+constexpr int kHeadDim = 128;
+constexpr int kAttnChunk = 32;      // cache positions per CTA
+constexpr int kAttnThreads = 256;
+constexpr int kRowPad = kHeadDim + 4;  // fp32 row stride in shared memory (16-byte rows, fewer conflicts)
+constexpr int kMaxT = 32;           // new tokens per sequence and call
+// Per-query partial record in the workspace: (max, sum, 2 unused, o[D]):
+// 132 floats = 528 bytes, so records and their o[] stay 16-byte aligned.
+constexpr int kPartStride = kHeadDim + 4;
+constexpr int kPartO = 4;
+
+// ---- RMSNorm -----------------------------------------------------------------
+__global__ void __launch_bounds__(256) rmsnorm_kernel(const __half* __restrict__ x,
+                                                      const __half* __restrict__ gamma, int64_t H,
+                                                      float eps, __half* __restrict__ y) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ float red[8];
+  const int64_t m = blockIdx.x;
+  const __half* xr = x + m * H;
+  float ss = 0.0f;
+  for (int64_t h = threadIdx.x; h < H; h += blockDim.x) {
+    const float v = __half2float(xr[h]);
+    ss = fmaf(v, v, ss);
+  }
+  ss = warp_sum(ss);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  float t = 0.0f;
+  for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+  const float r = 1.0f / sqrtf(t / (float)H + eps);
+  for (int64_t h = threadIdx.x; h < H; h += blockDim.x)
+    y[m * H + h] = __float2half_rn(__half2float(xr[h]) * r * __half2float(gamma[h]));
+}
+
+// ---- RoPE --------------------------------------------------------------------
+// Inverse frequencies theta^(-2d/D), d < D/2, computed on the host in fp64.
+struct RopeFreq {
+  double f[kHeadDim / 2];
+};
+
+// cos and sin of pos * f: the angle and its reduction modulo 2 pi in fp64
+// (positions up to 2^20 keep the reduced angle within ~1e-10), then fp32
+// sincosf of the reduced angle.
+__device__ __forceinline__ float2 rope_cs(int pos, double f) {
+  const double a = (double)pos * f;
+  const double k = rint(a * 0.15915494309189535);       // a / (2 pi)
+  double r = fma(-k, 6.283185307179586, a);              // 2 pi, head
+  r = fma(-k, 2.4492935982947064e-16, r);                 // 2 pi, tail
+  float s, c;
+  sincosf((float)r, &s, &c);
+  return make_float2(c, s);
+}
+
+// One CTA per (token row, key/value head): rotate the new key, copy the
+// value, both into the caches at the token's position.
+__global__ void __launch_bounds__(64) kv_append_kernel(const __half* __restrict__ qkv, int T, int Hq,
+                                                       int Hkv, const int32_t* __restrict__ pos0,
+                                                       const RopeFreq rf, __half* __restrict__ kc,
+                                                       __half* __restrict__ vc, int64_t max_ctx) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int row = blockIdx.x, h = blockIdx.y;
+  const int b = row / T, t = row - b * T;
+  const int pos = pos0[b] + t;
+  if (pos < 0 || (int64_t)pos >= max_ctx) {
+    if (threadIdx.x == 0) atomicOr(&g_attn_status, SQ_DEV_BAD_POSITION);
+    return;
+  }
+  const int64_t width = (int64_t)(Hq + 2 * Hkv) * kHeadDim;
+  const __half* kr = qkv + row * width + (int64_t)(Hq + h) * kHeadDim;
+  const __half* vr = qkv + row * width + (int64_t)(Hq + Hkv + h) * kHeadDim;
+  const int64_t dst = (((int64_t)b * Hkv + h) * max_ctx + pos) * kHeadDim;
+  const int d = threadIdx.x;  // pair (d, d + D/2)
+  const float2 cs = rope_cs(pos, rf.f[d]);
+  const float c = cs.x, s = cs.y;
+  const float x1 = __half2float(kr[d]), x2 = __half2float(kr[d + kHeadDim / 2]);
+  kc[dst + d] = __float2half_rn(x1 * c - x2 * s);
+  kc[dst + d + kHeadDim / 2] = __float2half_rn(x2 * c + x1 * s);
+  vc[dst + d] = vr[d];
+  vc[dst + d + kHeadDim / 2] = vr[d + kHeadDim / 2];
+}
+
+// ---- attention ----------------------------------------------------------------
+struct AttnArgs {
+  const __half* qkv;
+  const __half* kc;
+  const __half* vc;
+  const int32_t* pos0;
+  __half* out;
+  float* part;  // [(B*Hkv) * nsplit * Q * kPartStride]: per query (m, l, -, -, o[D])
+  int B, T, Hq, Hkv, G, Q;
+  int64_t max_ctx;
+  int nsplit;
+  float scale;  // 1 / sqrt(D)
+  RopeFreq rf;
+};
+
+// Shared memory (fp32): cos/sin of the T positions [T][D/2], q [Q][kRowPad]
+// (rotated, scaled), k [C][kRowPad], v [C][kRowPad], scores [Q][C].
+// Queries q = g * T + t (head kvh * G + g, token t).
+__global__ void __launch_bounds__(kAttnThreads) attention_partial_kernel(const AttnArgs a) {
+  griddep_wait();
+  griddep_launch_dependents();
+  extern __shared__ __align__(16) float sm[];
+  const int Q = a.Q, T = a.T;
+  float2* cst = reinterpret_cast<float2*>(sm);                  // [T][D/2]
+  float* qs = sm + 2 * kMaxT * (kHeadDim / 2);                  // [Q][kRowPad]
+  float* ks = qs + Q * kRowPad;                                 // [C][kRowPad]
+  float* vs = ks + kAttnChunk * kRowPad;                        // [C][kRowPad]
+  float* sc = vs + kAttnChunk * kRowPad;                        // [Q][C]
+  const int bh = blockIdx.x, split = blockIdx.y;
+  const int b = bh / a.Hkv, kvh = bh - b * a.Hkv;
+  const int tid = threadIdx.x;
+  const int p0 = a.pos0[b];
+  const int64_t len = (int64_t)p0 + T;  // cache entries after the append
+  const int64_t j0 = (int64_t)split * kAttnChunk;
+  float* part = a.part + ((int64_t)bh * a.nsplit + split) * Q * kPartStride;
+  if (j0 >= len || p0 < 0 || len > a.max_ctx) {  // empty chunk: neutral partials
+    for (int q = tid; q < Q; q += kAttnThreads) {
+      part[(int64_t)q * kPartStride] = -INFINITY;
+      part[(int64_t)q * kPartStride + 1] = 0.0f;
+    }
+    return;
+  }
+  const int nk = (int)(len - j0 < kAttnChunk ? len - j0 : kAttnChunk);
+  const int64_t width = (int64_t)(a.Hq + 2 * a.Hkv) * kHeadDim;
+  for (int idx = tid; idx < T * (kHeadDim / 2); idx += kAttnThreads) {
+    const int t = idx / (kHeadDim / 2), d = idx - t * (kHeadDim / 2);
+    cst[idx] = rope_cs(p0 + t, a.rf.f[d]);
+  }
+  const int64_t cbase = (((int64_t)b * a.Hkv + kvh) * a.max_ctx + j0) * kHeadDim;
+  for (int idx = tid; idx < kAttnChunk * kHeadDim; idx += kAttnThreads) {
+    const int j = idx / kHeadDim, d = idx - j * kHeadDim;
+    const bool in = j < nk;
+    ks[j * kRowPad + d] = in ? __half2float(a.kc[cbase + idx]) : 0.0f;
+    vs[j * kRowPad + d] = in ? __half2float(a.vc[cbase + idx]) : 0.0f;
+  }
+  __syncthreads();
+  for (int idx = tid; idx < Q * (kHeadDim / 2); idx += kAttnThreads) {
+    const int q = idx / (kHeadDim / 2), d = idx - q * (kHeadDim / 2);
+    const int g = q / T, t = q - g * T;
+    const __half* qr = a.qkv + ((int64_t)b * T + t) * width + (int64_t)(kvh * a.G + g) * kHeadDim;
+    const float2 cs = cst[t * (kHeadDim / 2) + d];
+    const float x1 = __half2float(qr[d]), x2 = __half2float(qr[d + kHeadDim / 2]);
+    qs[q * kRowPad + d] = (x1 * cs.x - x2 * cs.y) * a.scale;
+    qs[q * kRowPad + d + kHeadDim / 2] = (x2 * cs.x + x1 * cs.y) * a.scale;
+  }
+  __syncthreads();
+  // scores: each thread a 2-query x 4-key tile, 16-byte shared loads along D
+  const int qpairs = (Q + 1) / 2;
+  for (int tile = tid; tile < qpairs * (kAttnChunk / 4); tile += kAttnThreads) {
+    const int qp = tile / (kAttnChunk / 4), kq = tile - qp * (kAttnChunk / 4);
+    const int q0 = 2 * qp, q1 = q0 + 1 < Q ? q0 + 1 : q0;
+    float acc[2][4] = {};
+    const float4* qa = reinterpret_cast<const float4*>(qs + q0 * kRowPad);
+    const float4* qb = reinterpret_cast<const float4*>(qs + q1 * kRowPad);
+#pragma unroll 4
+    for (int d4 = 0; d4 < kHeadDim / 4; ++d4) {
+      const float4 x0 = qa[d4], x1 = qb[d4];
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+        const float4 kv = reinterpret_cast<const float4*>(ks + (4 * kq + kk) * kRowPad)[d4];
+        acc[0][kk] = fmaf(x0.x, kv.x, fmaf(x0.y, kv.y, fmaf(x0.z, kv.z, fmaf(x0.w, kv.w, acc[0][kk]))));
+        acc[1][kk] = fmaf(x1.x, kv.x, fmaf(x1.y, kv.y, fmaf(x1.z, kv.z, fmaf(x1.w, kv.w, acc[1][kk]))));
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int q = i ? q1 : q0;
+      if (i && q1 == q0) break;
+      const int t = q % T;
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+        const int j = 4 * kq + kk;
+        sc[q * kAttnChunk + j] = (j < nk && j0 + j <= (int64_t)p0 + t) ? acc[i][kk] : -INFINITY;
+      }
+    }
+  }
+  __syncthreads();
+  // per query: chunk max, exp, sum (one warp per query, one key per lane)
+  static_assert(kAttnChunk == 32, "one key per lane");
+  const int warp = tid >> 5, lane = tid & 31;
+  for (int q = warp; q < Q; q += kAttnThreads / 32) {
+    const float v = sc[q * kAttnChunk + lane];
+    const float mx = warp_max(v);
+    const float e = mx == -INFINITY ? 0.0f : expf(v - mx);
+    sc[q * kAttnChunk + lane] = e;
+    const float l = warp_sum(e);
+    if (lane == 0) {
+      part[(int64_t)q * kPartStride] = mx;
+      part[(int64_t)q * kPartStride + 1] = l;
+    }
+  }
+  __syncthreads();
+  // weighted values: each thread a 2-query x 4-dim tile
+  for (int tile = tid; tile < qpairs * (kHeadDim / 4); tile += kAttnThreads) {
+    const int qp = tile / (kHeadDim / 4), d4 = tile - qp * (kHeadDim / 4);
+    const int q0 = 2 * qp, q1 = q0 + 1 < Q ? q0 + 1 : q0;
+    float4 o0 = make_float4(0.f, 0.f, 0.f, 0.f), o1 = o0;
+    for (int j = 0; j < nk; ++j) {
+      const float e0 = sc[q0 * kAttnChunk + j], e1 = sc[q1 * kAttnChunk + j];
+      const float4 vv = reinterpret_cast<const float4*>(vs + j * kRowPad)[d4];
+      o0.x = fmaf(e0, vv.x, o0.x); o0.y = fmaf(e0, vv.y, o0.y);
+      o0.z = fmaf(e0, vv.z, o0.z); o0.w = fmaf(e0, vv.w, o0.w);
+      o1.x = fmaf(e1, vv.x, o1.x); o1.y = fmaf(e1, vv.y, o1.y);
+      o1.z = fmaf(e1, vv.z, o1.z); o1.w = fmaf(e1, vv.w, o1.w);
+    }
+    *reinterpret_cast<float4*>(part + (int64_t)q0 * kPartStride + kPartO + 4 * d4) = o0;
+    if (q1 != q0) *reinterpret_cast<float4*>(part + (int64_t)q1 * kPartStride + kPartO + 4 * d4) = o1;
+  }
+}
+
+// One CTA per (sequence and key/value head, query): the chunk maxima and
+// sums are read in parallel into shared memory, then each thread (one per
+// head dimension) merges the chunks' weighted values.
+__global__ void __launch_bounds__(kHeadDim) attention_combine_kernel(const AttnArgs a) {
+  griddep_wait();
+  griddep_launch_dependents();
+  extern __shared__ float cm[];  // [2 * nsplit]: chunk max, chunk sum
+  __shared__ float red[kHeadDim / 32];
+  const int bh = blockIdx.x, q = blockIdx.y, d = threadIdx.x;
+  const int b = bh / a.Hkv, kvh = bh - b * a.Hkv;
+  const float* base = a.part + (int64_t)bh * a.nsplit * a.Q * kPartStride;
+  float M = -INFINITY;
+  for (int s = d; s < a.nsplit; s += kHeadDim) {
+    const float* ps = base + ((int64_t)s * a.Q + q) * kPartStride;
+    cm[s] = ps[0];
+    cm[a.nsplit + s] = ps[1];
+    M = fmaxf(M, ps[0]);
+  }
+  M = warp_max(M);
+  if ((d & 31) == 0) red[d >> 5] = M;
+  __syncthreads();
+  M = -INFINITY;
+#pragma unroll
+  for (int w = 0; w < kHeadDim / 32; ++w) M = fmaxf(M, red[w]);
+  float L = 0.0f, O = 0.0f;
+  if (M != -INFINITY)
+    for (int s = 0; s < a.nsplit; ++s) {
+      const float ms = cm[s];
+      if (ms == -INFINITY) continue;
+      const float w = expf(ms - M);
+      L = fmaf(w, cm[a.nsplit + s], L);
+      O = fmaf(w, base[((int64_t)s * a.Q + q) * kPartStride + kPartO + d], O);
+    }
+  const int g = q / a.T, t = q - g * a.T;
+  const int64_t row = (int64_t)b * a.T + t;
+  a.out[row * (int64_t)a.Hq * kHeadDim + (int64_t)(kvh * a.G + g) * kHeadDim + d] =
+      __float2half_rn(L > 0.0f ? O / L : 0.0f);
+}
+
+// ---- rollback -------------------------------------------------------------------
+__global__ void kv_rollback_kernel(const int32_t* __restrict__ base, const int32_t* __restrict__ n,
+                                   int B, int limit, int32_t* __restrict__ len) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  const int na = n[b];
+  len[b] = na < 0 ? base[b] : base[b] + (na + 1 < limit ? na + 1 : limit);
+}
+
+// ---- host side -------------------------------------------------------------------
+cudaError_t launch_rmsnorm(const __half* x, const __half* gamma, int M, int64_t H, float eps, __half* y,
+                           cudaStream_t st) {
+  if (M == 0) return cudaSuccess;
+  return launch_pdl(rmsnorm_kernel, dim3((unsigned)M), dim3(256), 0, st, x, gamma, H, eps, y);
+}
+
+static RopeFreq rope_freq(double theta) {
+  RopeFreq rf;
+  for (int d = 0; d < kHeadDim / 2; ++d) rf.f[d] = pow(theta, -2.0 * d / (double)kHeadDim);
+  return rf;
+}
+
+cudaError_t launch_kv_append(const __half* qkv, int B, int T, int Hq, int Hkv, const int32_t* pos0,
+                             double theta, __half* kc, __half* vc, int64_t max_ctx, cudaStream_t st) {
+  if (B == 0 || T == 0) return cudaSuccess;
+  return launch_pdl(kv_append_kernel, dim3((unsigned)(B * T), (unsigned)Hkv), dim3(kHeadDim / 2), 0, st,
+                    qkv, T, Hq, Hkv, pos0, rope_freq(theta), kc, vc, max_ctx);
+}
+
+size_t attention_workspace_bytes(int B, int T, int Hq, int Hkv, int64_t max_ctx) {
+  if (B < 0 || T < 0 || Hkv <= 0 || max_ctx <= 0) return 0;
+  const int64_t nsplit = (max_ctx + kAttnChunk - 1) / kAttnChunk;
+  const int64_t Q = (int64_t)(Hq / Hkv) * T;
+  return (size_t)B * Hkv * nsplit * Q * kPartStride * sizeof(float);
+}
+
+size_t attention_smem_bytes(int Q) {
+  return ((size_t)2 * kMaxT * (kHeadDim / 2) + (size_t)Q * kRowPad + (size_t)2 * kAttnChunk * kRowPad +
+          (size_t)Q * kAttnChunk) * sizeof(float);
+}
+
+int attention_max_tokens() { return kMaxT; }
+
+cudaError_t launch_attention(const __half* qkv, int B, int T, int Hq, int Hkv, const int32_t* pos0,
+                             double theta, const __half* kc, const __half* vc, int64_t max_ctx,
+                             __half* out, void* ws, cudaStream_t st) {
+  if (B == 0 || T == 0) return cudaSuccess;
+  AttnArgs a = {};
+  a.qkv = qkv;
+  a.kc = kc;
+  a.vc = vc;
+  a.pos0 = pos0;
+  a.out = out;
+  a.part = reinterpret_cast<float*>(ws);
+  a.B = B;
+  a.T = T;
+  a.Hq = Hq;
+  a.Hkv = Hkv;
+  a.G = Hq / Hkv;
+  a.Q = a.G * T;
+  a.max_ctx = max_ctx;
+  a.nsplit = (int)((max_ctx + kAttnChunk - 1) / kAttnChunk);
+  a.rf = rope_freq(theta);
+  a.scale = 1.0f / sqrtf((float)kHeadDim);
+  const size_t smem = attention_smem_bytes(a.Q);
+  static int smem_set[64] = {0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if ((int)smem > smem_set[dev]) {
+    e = cudaFuncSetAttribute(attention_partial_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    smem_set[dev] = (int)smem;
+  }
+  e = launch_pdl(attention_partial_kernel, dim3((unsigned)(B * Hkv), (unsigned)a.nsplit),
+                 dim3(kAttnThreads), smem, st, a);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(attention_combine_kernel, dim3((unsigned)(B * Hkv), (unsigned)a.Q), dim3(kHeadDim),
+                    (size_t)2 * a.nsplit * sizeof(float), st, a);
+}
+
+cudaError_t launch_kv_rollback(const int32_t* base, const int32_t* n, int B, int limit, int32_t* len,
+                               cudaStream_t st) {
+  if (B == 0) return cudaSuccess;
+  return launch_pdl(kv_rollback_kernel, dim3((unsigned)((B + 127) / 128)), dim3(128), 0, st, base, n, B,
+                    limit, len);
+}
+
+cudaError_t take_attn_status(uint32_t* bits) {
+  uint32_t v = 0, zero = 0;
+  cudaError_t e = cudaMemcpyFromSymbol(&v, g_attn_status, sizeof(v));
+  if (e != cudaSuccess) return e;
+  if (v) e = cudaMemcpyToSymbol(g_attn_status, &zero, sizeof(zero));
+  *bits |= v;
+  return e;
+}
+
+}  // namespace sq

@@ -62,7 +62,8 @@ sq_status sq_check(sq_stream_t stream, uint32_t* device_bits) {
   if ((e = take_accept_status(&bits)) != cudaSuccess) return cuda_fail(e, "sq_check: accept status");
   if ((e = take_gemv_status_int4(&bits)) != cudaSuccess ||
       (e = take_gemv_status_fp8(&bits)) != cudaSuccess ||
-      (e = take_gemv_status_fp16(&bits)) != cudaSuccess || (e = take_tc_status(&bits)) != cudaSuccess)
+      (e = take_gemv_status_fp16(&bits)) != cudaSuccess || (e = take_tc_status(&bits)) != cudaSuccess ||
+      (e = take_attn_status(&bits)) != cudaSuccess)
     return cuda_fail(e, "sq_check: linear status");
   if (device_bits) *device_bits = bits;
   if (bits) return fail(SQ_ERR_DEVICE, "sq_check: device status bits 0x%x", bits);
@@ -397,6 +398,88 @@ sq_status sq_softmax(const void* z, int64_t R, int64_t V, float temperature, flo
   softmax_layout(sa, workspace);
   cudaError_t e = launch_softmax(sa, p, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "sq_softmax: launch");
+  return SQ_OK;
+}
+
+// ---- decoder pieces
+
+sq_status sq_rmsnorm(const void* x, const void* gamma, int M, int64_t H, float eps, void* y,
+                     sq_stream_t stream) {
+  if (M < 0 || H < 1) return fail(SQ_ERR_SHAPE, "sq_rmsnorm: need M >= 0, H >= 1");
+  if (!(eps >= 0.0f) || !std::isfinite(eps)) return fail(SQ_ERR_INVALID_ARG, "sq_rmsnorm: bad eps");
+  if (M == 0) return SQ_OK;
+  if (!x || !gamma || !y) return fail(SQ_ERR_INVALID_ARG, "sq_rmsnorm: NULL pointer");
+  if (!aligned(x, 2) || !aligned(gamma, 2) || !aligned(y, 2))
+    return fail(SQ_ERR_ALIGN, "sq_rmsnorm: pointers must be 2-byte aligned");
+  cudaError_t e = launch_rmsnorm(reinterpret_cast<const __half*>(x), reinterpret_cast<const __half*>(gamma),
+                                 M, H, eps, reinterpret_cast<__half*>(y), (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_rmsnorm: launch");
+  return SQ_OK;
+}
+
+static sq_status check_attn(const char* who, const void* qkv, int B, int T, int Hq, int Hkv, int D,
+                            const int32_t* pos0, float theta, const void* kc, const void* vc,
+                            int64_t max_ctx) {
+  if (B < 0 || T < 0 || Hq < 1 || Hkv < 1 || Hq % Hkv || max_ctx < 1)
+    return fail(SQ_ERR_SHAPE, "%s: need B, T >= 0, Hq a positive multiple of Hkv, max_ctx >= 1", who);
+  if (D != 128) return fail(SQ_ERR_UNSUPPORTED, "%s: head dimension %d (only 128 is built)", who, D);
+  if ((Hq / Hkv) * T > 200 || T > attention_max_tokens())
+    return fail(SQ_ERR_SHAPE, "%s: need (Hq / Hkv) * T <= 200 and T <= %d", who, attention_max_tokens());
+  if (!(theta > 1.0f) || !std::isfinite(theta)) return fail(SQ_ERR_INVALID_ARG, "%s: theta must be > 1", who);
+  if (B > 0 && T > 0 && (!qkv || !pos0 || !kc || !vc))
+    return fail(SQ_ERR_INVALID_ARG, "%s: NULL pointer", who);
+  if (!aligned(qkv, 2) || !aligned(pos0, 4) || !aligned(kc, 2) || !aligned(vc, 2))
+    return fail(SQ_ERR_ALIGN, "%s: misaligned pointer", who);
+  return SQ_OK;
+}
+
+sq_status sq_kv_append(const void* qkv, int B, int T, int Hq, int Hkv, int D, const int32_t* pos0,
+                       float theta, void* k_cache, void* v_cache, int64_t max_ctx, sq_stream_t stream) {
+  sq_status st = check_attn("sq_kv_append", qkv, B, T, Hq, Hkv, D, pos0, theta, k_cache, v_cache, max_ctx);
+  if (st != SQ_OK) return st;
+  cudaError_t e = launch_kv_append(reinterpret_cast<const __half*>(qkv), B, T, Hq, Hkv, pos0, (double)theta,
+                                   reinterpret_cast<__half*>(k_cache), reinterpret_cast<__half*>(v_cache),
+                                   max_ctx, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_kv_append: launch");
+  return SQ_OK;
+}
+
+size_t sq_attention_workspace_bytes(int B, int T, int Hq, int Hkv, int D, int64_t max_ctx) {
+  if (D != 128 || Hkv < 1 || Hq % Hkv) return 0;
+  return attention_workspace_bytes(B, T, Hq, Hkv, max_ctx);
+}
+
+sq_status sq_attention(const void* qkv, int B, int T, int Hq, int Hkv, int D, const int32_t* pos0,
+                       float theta, const void* k_cache, const void* v_cache, int64_t max_ctx, void* out,
+                       void* workspace, size_t ws_bytes, sq_stream_t stream) {
+  sq_status st = check_attn("sq_attention", qkv, B, T, Hq, Hkv, D, pos0, theta, k_cache, v_cache, max_ctx);
+  if (st != SQ_OK) return st;
+  if (B == 0 || T == 0) return SQ_OK;
+  if (!out || !aligned(out, 2)) return fail(SQ_ERR_ALIGN, "sq_attention: out NULL or misaligned");
+  const size_t need = attention_workspace_bytes(B, T, Hq, Hkv, max_ctx);
+  if (!workspace || ws_bytes < need)
+    return fail(SQ_ERR_WORKSPACE, "sq_attention: workspace %zu bytes < %zu required", ws_bytes, need);
+  if (!aligned(workspace, 16)) return fail(SQ_ERR_ALIGN, "sq_attention: workspace must be 16-byte aligned");
+  if (attention_smem_bytes((Hq / Hkv) * T) > (size_t)device_max_smem())
+    return fail(SQ_ERR_SHAPE, "sq_attention: query group too large for shared memory");
+  if (max_ctx > ((int64_t)1 << 17)) return fail(SQ_ERR_SHAPE, "sq_attention: max_ctx > 2^17");
+  cudaError_t e = launch_attention(reinterpret_cast<const __half*>(qkv), B, T, Hq, Hkv, pos0, (double)theta,
+                                   reinterpret_cast<const __half*>(k_cache),
+                                   reinterpret_cast<const __half*>(v_cache), max_ctx,
+                                   reinterpret_cast<__half*>(out), workspace, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_attention: launch");
+  return SQ_OK;
+}
+
+sq_status sq_kv_rollback(const int32_t* base, const int32_t* n_accepted, int B, int limit, int32_t* len,
+                         sq_stream_t stream) {
+  if (B < 0 || limit < 0) return fail(SQ_ERR_SHAPE, "sq_kv_rollback: need B >= 0, limit >= 0");
+  if (B == 0) return SQ_OK;
+  if (!base || !n_accepted || !len) return fail(SQ_ERR_INVALID_ARG, "sq_kv_rollback: NULL pointer");
+  if (!aligned(base, 4) || !aligned(n_accepted, 4) || !aligned(len, 4))
+    return fail(SQ_ERR_ALIGN, "sq_kv_rollback: pointers must be 4-byte aligned");
+  cudaError_t e = launch_kv_rollback(base, n_accepted, B, limit, len, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_kv_rollback: launch");
   return SQ_OK;
 }
 

@@ -167,3 +167,74 @@ def run_pass_unchained(stack: LinearStack, variant: str, b: PassBuffers, stream=
     """The same pass as separate sq_linear_ex calls."""
     for (wk, x, w, s, bias, res, epi, y) in pass_ops(stack, variant, b, logits):
         sq_linear_ex(wk, x, w, s, bias, res, epi, y, stream)
+
+
+# ---- the decoder step around the linear stack ---------------------------------------
+
+HEAD_DIM = 128
+ROPE_THETA = 1e6       # Qwen2.5
+RMS_EPS = 1e-6
+
+
+class DecoderState:
+    """Per-model state of a decoder pass over T new tokens of B sequences: a
+    KV cache per layer ([B, Hkv, max_ctx, 128] fp16, keys rotated), the
+    RMSNorm gains, the residual stream and the pass's activations.  Token t
+    of sequence b sits at position pos0[b] + t."""
+
+    def __init__(self, stack: LinearStack, B: int, T: int, max_ctx: int, context: int,
+                 seed: int = 5):
+        from . import sq_attention_workspace_bytes
+        sh, dev = stack.shape, stack.device
+        self.B, self.T, self.max_ctx = B, T, max_ctx
+        nl = len(stack.layers)
+        cache = (B, sh.kv_heads, max_ctx, HEAD_DIM)
+        self.k = [torch.zeros(cache, dtype=torch.float16, device=dev) for _ in range(nl)]
+        self.v = [torch.zeros(cache, dtype=torch.float16, device=dev) for _ in range(nl)]
+        g = [1.0 + synth.fp16_normal(seed + i, (sh.hidden,), 0.05).astype("float32")
+             for i in range(2 * nl + 1)]
+        self.gamma = [torch.from_numpy(a.astype("float16")).to(dev) for a in g]
+        self.pos0 = torch.full((B,), context, dtype=torch.int32, device=dev)
+        M = B * T
+        self.x = synth.activations_fp16_device(seed + 99, M, sh.hidden, dev)
+        self.h = torch.empty((M, sh.hidden), dtype=torch.float16, device=dev)
+        self.qkv = torch.empty((M, sh.q_out + 2 * sh.kv_out), dtype=torch.float16, device=dev)
+        self.attn = torch.empty((M, sh.q_out), dtype=torch.float16, device=dev)
+        self.g = torch.empty((M, sh.intermediate), dtype=torch.float16, device=dev)
+        self.logits = torch.empty((M, sh.vocab), dtype=torch.float16, device=dev) \
+            if stack.lm_head is not None else None
+        self.ws = torch.empty(sq_attention_workspace_bytes(B, T, sh.q_heads, sh.kv_heads, max_ctx),
+                              dtype=torch.uint8, device=dev)
+
+
+def decoder_pass(stack: LinearStack, variant: str, st: DecoderState, stream=None,
+                 logits=None) -> None:
+    """One decoder step (draft or verify) with the variant's weights: per
+    layer x += o(attn(rope(qkv(norm(x))))), x += down(silu-gate(norm(x)));
+    then logits = lm_head(norm(x)) (into `logits` when given).  The new
+    tokens' keys and values are appended to the caches before attention
+    reads them."""
+    from . import SQ_EPI_RESIDUAL, sq_attention, sq_kv_append, sq_rmsnorm
+    sh = stack.shape
+    wk = WKIND[variant]
+    B, T = st.B, st.T
+    for li, (qkv, o, gu, down) in enumerate(stack.layers):
+        sq_rmsnorm(st.x, st.gamma[2 * li], RMS_EPS, st.h, stream)
+        w, s = qkv.weight(variant)
+        sq_linear_ex(wk, st.h, w, s, None, None, SQ_EPI_NONE, st.qkv, stream)
+        sq_kv_append(st.qkv, B, T, sh.q_heads, sh.kv_heads, st.pos0, ROPE_THETA, st.k[li], st.v[li],
+                     stream)
+        sq_attention(st.qkv, B, T, sh.q_heads, sh.kv_heads, st.pos0, ROPE_THETA, st.k[li], st.v[li],
+                     st.attn, st.ws, stream)
+        w, s = o.weight(variant)
+        sq_linear_ex(wk, st.attn, w, s, None, st.x, SQ_EPI_RESIDUAL, st.x, stream)
+        sq_rmsnorm(st.x, st.gamma[2 * li + 1], RMS_EPS, st.h, stream)
+        w, s = gu.weight(variant)
+        sq_linear_ex(wk, st.h, w, s, None, None, SQ_EPI_SILU_GATE, st.g, stream)
+        w, s = down.weight(variant)
+        sq_linear_ex(wk, st.g, w, s, None, st.x, SQ_EPI_RESIDUAL, st.x, stream)
+    if stack.lm_head is not None:
+        sq_rmsnorm(st.x, st.gamma[-1], RMS_EPS, st.h, stream)
+        w, s = stack.lm_head.weight(variant)
+        sq_linear_ex(wk, st.h, w, s, None, None, SQ_EPI_NONE, st.logits if logits is None else logits,
+                     stream)
