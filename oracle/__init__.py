@@ -363,3 +363,118 @@ def attention(q, k, v, qpos) -> np.ndarray:
     out = np.empty((T, Hq, D), np.float64)
     _load().oq_attention(_ptr(qa), _ptr(ka), _ptr(va), _ptr(pa), T, L, Hq, Hkv, D, _ptr(out))
     return out
+
+
+def silu_gate_rows(gu, inter: int) -> np.ndarray:
+    """silu(g) * u for rows gu = [g | u] of width 2 * inter (the fused gate/up layout)."""
+    gu = np.asarray(gu, np.float64)
+    return silu_gate(gu[:, :inter], gu[:, inter:])
+
+
+# ---- Sec. III-D: the decoder as a function of its token sequence -----------------
+#
+# A plain restatement with no KV cache: every call recomputes the whole
+# sequence, so the cache, its positions and its rollback on the CUDA side are
+# checked against a computation that has none of them.  Model internals follow
+# the Qwen2.5 decoder (the paper gives none): pre-norm layers
+#   x += o(attention(rope(q), rope(k), v)),  x += down(silu(gate) * up)
+# over RMSNorm'ed inputs, a final RMSNorm and the lm_head; the input
+# embedding is its own fp16 table (or the lm_head's, tied, when absent).
+
+def decoder_logits(params: dict, tokens, rows=None) -> np.ndarray:
+    """Logits (fp64) of the decoder over one token sequence.
+
+    params: 'layers' = list of (w_qkv, w_o, w_gate_up, w_down) float arrays,
+    'lm_head' [V, H], 'embed' [V, H] (optional), 'gamma' = 2 L + 1 gains, 'q_heads', 'kv_heads',
+    'head_dim', 'intermediate', 'eps', 'theta'.  rows: positions whose
+    logits are wanted (default: all)."""
+    tok = np.asarray(tokens, np.int64)
+    n = len(tok)
+    Hq, Hkv, D = params["q_heads"], params["kv_heads"], params["head_dim"]
+    inter, eps, theta = params["intermediate"], params["eps"], params["theta"]
+    emb = np.asarray(params.get("embed", params["lm_head"]), np.float64)
+    lm = np.asarray(params["lm_head"], np.float64)
+    gam = params["gamma"]
+    pos = np.arange(n, dtype=np.int64)
+    x = emb[tok].copy()
+    for li, (w_qkv, w_o, w_gu, w_dn) in enumerate(params["layers"]):
+        h = rmsnorm(x, gam[2 * li], eps)
+        qkv = linear(h, w_qkv)
+        q = rope(qkv[:, :Hq * D], pos, Hq, D, theta)
+        k = rope(qkv[:, Hq * D:(Hq + Hkv) * D], pos, Hkv, D, theta)
+        v = qkv[:, (Hq + Hkv) * D:]
+        a = attention(q.reshape(n, Hq, D), k.reshape(n, Hkv, D), v.reshape(n, Hkv, D), pos)
+        x = x + linear(a.reshape(n, Hq * D), w_o)
+        h = rmsnorm(x, gam[2 * li + 1], eps)
+        x = x + linear(silu_gate_rows(linear(h, w_gu), inter), w_dn)
+    sel = pos if rows is None else np.asarray(rows, np.int64)
+    return linear(rmsnorm(x[sel], gam[-1], eps), lm)
+
+
+def generate_greedy(params: dict, prompt, n_new: int):
+    """Greedy continuation of one prompt: each new token is the argmax of
+    the logits at the last position given everything before it (lowest
+    index on ties).  Returns (tokens, gaps), gaps[i] = the distance between
+    the two largest logits at step i (how far step i is from a tie)."""
+    seq = [int(t) for t in prompt]
+    out, gaps = [], []
+    for _ in range(n_new):
+        z = decoder_logits(params, seq, rows=[len(seq) - 1])[0]
+        order = np.argsort(-z, kind="stable")
+        out.append(int(order[0]))
+        gaps.append(float(z[order[0]] - z[order[1]]))
+        seq.append(int(order[0]))
+    return out, gaps
+
+
+# ---- Sec. III-D.4: the bookkeeping between cycles --------------------------------
+
+def spec_commit(n_accepted, tokens, hist, length, K: int):
+    """Append tokens[b, :n+1] (n = n_accepted[b]; None = 0; n < 0 appends
+    nothing) to each history, then the next cycle's positions pos [K+1, B]
+    (draft step 0 at L-2, draft step k at L-1+k, verify at L-1) and the last
+    two tokens.  Returns (hist, length, pos, last2, bad) as new arrays;
+    `bad` marks a sequence whose history overflowed or is shorter than 2."""
+    hist = [list(map(int, h)) for h in np.asarray(hist)]
+    length = [int(x) for x in np.asarray(length)]
+    tokens = np.asarray(tokens).reshape(len(length), -1)
+    B, cap = len(length), len(hist[0])
+    pos = np.zeros((K + 1, B), np.int32)
+    last2 = np.zeros((B, 2), np.int32)
+    bad = np.zeros(B, bool)
+    for b in range(B):
+        L = length[b]
+        if L < 0 or L > cap:
+            bad[b], L = True, 0
+        else:
+            n = 0 if n_accepted is None else int(n_accepted[b])
+            if n >= tokens.shape[1]:
+                bad[b] = True
+            elif n >= 0:
+                new = [int(t) for t in tokens[b, :n + 1]]
+                room = cap - L
+                if len(new) > room:
+                    bad[b] = True
+                    new = new[:room]
+                hist[b][L:L + len(new)] = new
+                L += len(new)
+        if L < 2:
+            bad[b] = True
+        length[b] = L
+        last2[b] = (hist[b][L - 2] if L >= 2 else -1, hist[b][L - 1] if L >= 1 else -1)
+        if K >= 1:
+            pos[0, b] = L - 2
+        for k in range(1, K):
+            pos[k, b] = L - 1 + k
+        pos[K, b] = L - 1
+    return np.array(hist, np.int32), np.array(length, np.int32), pos, last2, bad
+
+
+def spec_drafts(samples, last2):
+    """(verify tokens [B, K+1], draft [B, K]) from the draft steps' tokens
+    samples [K, B] and the last committed token last2[:, 1]."""
+    s = np.asarray(samples, np.int32)
+    l2 = np.asarray(last2, np.int32)
+    K, B = s.shape
+    verify = np.concatenate([l2[:, 1:2], s.T], axis=1)
+    return verify.astype(np.int32), s.T.copy()

@@ -86,6 +86,25 @@ def spec_block(seed: int, B: int, K: int, V: int, sigma: float = 2.0,
     return p, q, draft, u
 
 
+def stack_weight_seed(seed: int, index: int) -> int:
+    """Seed of the index-th projection (decoder order, lm_head last) of a
+    linear stack built with base seed `seed`."""
+    return (seed + index) * 7919 + 17
+
+
+def rms_gains(seed: int, hidden: int, count: int) -> list:
+    """RMSNorm gains 1 + N(0, 0.05), rounded to fp16: two per decoder layer
+    (attention, MLP) and then the final norm."""
+    return [(1.0 + fp16_normal(seed + i, (hidden,), 0.05).astype(np.float32)).astype(np.float16)
+            for i in range(count)]
+
+
+def prompt_tokens(seed: int, B: int, P: int, vocab: int) -> np.ndarray:
+    """Synthetic prompts: int32 [B, P] token ids uniform over the vocabulary."""
+    z = splitmix64(seed ^ 0x70C0, np.arange(B * P, dtype=np.uint64))
+    return (z % np.uint64(vocab)).astype(np.int32).reshape(B, P)
+
+
 def weights_fp16_device(seed: int, n_out: int, k_in: int, device, std: float = 0.02):
     """Large fp16 ~ N(0, std) weight matrices drawn on the device with a
     seeded torch generator (used for full-size workloads; tests copy the
