@@ -479,6 +479,48 @@ def main():
         t_dc = timed(g_dc, reps_c) / reps_c
         t_ddir = timed(g_ddir, reps) / reps
         del g_dd, g_dv, g_dc, g_ddir, dd, dv
+
+        # whole greedy generations through the device-side cycle (embedding,
+        # decoder passes, draft argmax, accept, commit; one graph replay per
+        # cycle) from synthetic 32-token prompts: the acceptance the derived
+        # variant reaches against its parent on this random-init model, and
+        # speculative against direct tokens/s measured the same way
+        from paper_2609_21704_gb300.generate import Generator
+        gen_P, gen_cs, gen_cd = 32, 48, 96
+        prompts = synth.prompt_tokens(61 + rank, B, gen_P, V)
+
+        def gen_time(k, cycles):
+            g = Generator(stack, B, k, gen_P, gen_P + 1 + k + (cycles + 2) * (k + 1), draft=args.draft,
+                          seed=70 + rank)
+            g.prefill(prompts, stream)
+            g.run(2, stream)                    # eager cycle + capture, one replay
+            stream.synchronize()
+            l0 = g.len.cpu().numpy().copy()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            g.run(cycles, stream)
+            e1.record(stream)
+            e1.synchronize()
+            toks = g.tokens()
+            made = int((g.len.cpu().numpy() - l0).sum())
+            if g.status() != 0:
+                raise RuntimeError("generation flagged the device status word")
+            distinct = sum(len(set(t[gen_P:])) for t in toks) / B
+            return e0.elapsed_time(e1) / 1e3, made, distinct
+
+        t_gs, made_s, distinct_s = gen_time(K, gen_cs)
+        t_gd, made_d, _ = gen_time(0, gen_cd)
+        gen = {
+            "prompt_tokens": gen_P, "mode": "greedy", "cycles": gen_cs,
+            "tokens_per_cycle": made_s / (B * gen_cs),
+            "alpha_measured": (made_s / (B * gen_cs) - 1.0) / K,
+            "ms_per_cycle": 1e3 * t_gs / gen_cs,
+            "tokens_per_s": world * made_s / t_gs,
+            "direct_fp16_tokens_per_s": world * made_d / t_gd,
+            "speedup_vs_direct_fp16": (made_s / t_gs) / (made_d / t_gd),
+            "distinct_tokens_per_sequence": distinct_s,
+        }
     tensor_peak, tensor_peak_kind = measured_tensor_peak()
     pf_flops = 2.0 * 256 * stack.params()
     draft_bytes = stack.weight_bytes(args.draft) + stack.activation_bytes(B)
@@ -606,6 +648,7 @@ def main():
             "decoder_tokens_per_s": B * world * mean_tokens / t_dc,
             "decoder_direct_fp16_tokens_per_s": B * world / t_ddir,
             "decoder_speedup_vs_direct_fp16": (mean_tokens / t_dc) / (1.0 / t_ddir),
+            "generation": gen,
             "prefill_m256_fp16_ms": 1e3 * t_pf16,
             "prefill_m256_fp16_tflops": pf_flops / t_pf16 / 1e12,
             "prefill_m256_%s_ms" % args.draft: 1e3 * t_pfd,

@@ -76,6 +76,7 @@ typedef enum { SQ_ACCEPT_SAMPLE = 0, SQ_ACCEPT_GREEDY = 1 } sq_accept_mode;
 #define SQ_DEV_TIMEOUT          0x10u /* a kernel gave up a bounded wait     */
 #define SQ_DEV_NONFINITE_LOGIT  0x20u /* a logit row held inf or NaN         */
 #define SQ_DEV_BAD_POSITION     0x40u /* a token position outside the cache  */
+#define SQ_DEV_BAD_TOKEN_ID     0x80u /* an embedding id outside [0, V)      */
 
 /* Thread-local text of the last error raised on this host thread. */
 SQ_API const char* sq_last_error(void);
@@ -328,6 +329,37 @@ SQ_API sq_status sq_attention(const void* qkv, int B, int T, int Hq, int Hkv, in
                               size_t ws_bytes, sq_stream_t stream);
 SQ_API sq_status sq_kv_rollback(const int32_t* base, const int32_t* n_accepted, int B, int limit,
                                 int32_t* len, sq_stream_t stream);
+/* sq_embed: out[m, :] = table[ids[m * ids_stride], :] for M token ids
+ * (int32, device), table fp16 [V, H], out fp16 [M, H]; an id outside [0, V)
+ * gives a zero row and sets SQ_DEV_BAD_TOKEN_ID.  This is how accepted and
+ * drafted tokens re-enter the model (the same call gathers rows of any
+ * [rows, H] fp16 matrix).
+ *
+ * Speculative bookkeeping on the device, so that a whole draft / verify /
+ * accept cycle runs without the host (Sec. III-D.4: the accepted prefix plus
+ * the correction token is the context the next cycle starts from).  Per
+ * sequence b: hist int32 [B, cap] holds the committed tokens, len[b] of them.
+ *
+ * sq_spec_commit: appends tokens[b, 0 .. n] (n = n_accepted[b], or 0 when
+ *   n_accepted is NULL; row stride ldt; nothing when n < 0) to hist[b] and
+ *   adds them to len[b]; then, with L the new length, writes the next
+ *   cycle's positions pos int32 [K + 1, B]: pos[0, b] = L - 2 (the first
+ *   draft step feeds the last two committed tokens, T = 2), pos[k, b] =
+ *   L - 1 + k for draft steps k = 1 .. K-1 (T = 1), pos[K, b] = L - 1 (the
+ *   verify pass, T = K + 1; with K = 0 this is direct decoding); and
+ *   last2 int32 [B, 2] = (hist[b, L-2], hist[b, L-1]).  An overfull history,
+ *   n >= ldt, a length outside [0, cap] or L < 2 sets SQ_DEV_BAD_POSITION
+ *   (missing tokens read as -1).
+ * sq_spec_drafts: verify_tokens int32 [B, K+1] = (last2[b, 1], samples[0,b],
+ *   .., samples[K-1, b]) and draft int32 [B, K] = samples^T, from the K
+ *   draft steps' tokens samples int32 [K, B]. */
+SQ_API sq_status sq_embed(const int32_t* ids, int M, int64_t ids_stride, const void* table, int64_t V,
+                          int64_t H, void* out, sq_stream_t stream);
+SQ_API sq_status sq_spec_commit(const int32_t* n_accepted, const int32_t* tokens, int ldt, int B, int K,
+                                int32_t* hist, int cap, int32_t* len, int32_t* pos, int32_t* last2,
+                                sq_stream_t stream);
+SQ_API sq_status sq_spec_drafts(const int32_t* samples, const int32_t* last2, int B, int K,
+                                int32_t* verify_tokens, int32_t* draft, sq_stream_t stream);
 
 /* ------------------------------------------------------------------------
  * sq_accept_noalloc: sq_accept without a caller workspace.  The paper has

@@ -29,7 +29,8 @@ __all__ = [
     "sq_version", "sq_accept_noalloc", "sq_linear_path", "sq_linear_chain", "SqLinearOp",
     "sq_accept_logits_workspace_bytes", "sq_accept_logits", "sq_sample_logits",
     "sq_softmax_workspace_bytes", "sq_softmax", "sq_rmsnorm", "sq_kv_append",
-    "sq_attention_workspace_bytes", "sq_attention", "sq_kv_rollback",
+    "sq_attention_workspace_bytes", "sq_attention", "sq_kv_rollback", "sq_embed",
+    "sq_spec_commit", "sq_spec_drafts",
     "EXPORTED_SYMBOLS",
 ]
 
@@ -39,7 +40,7 @@ SQ_ACCEPT_SAMPLE, SQ_ACCEPT_GREEDY = 0, 1
 SQ_EPI_NONE, SQ_EPI_SILU_GATE, SQ_EPI_RESIDUAL = 0, 1, 2
 SQ_W_FP16, SQ_W_INT4, SQ_W_FP8 = 0, 1, 2
 SQ_DEV_NONFINITE_WEIGHT, SQ_DEV_BAD_DRAFT_TOKEN, SQ_DEV_NO_MASS, SQ_DEV_BAD_UNIFORM = 1, 2, 4, 8
-SQ_DEV_TIMEOUT, SQ_DEV_NONFINITE_LOGIT, SQ_DEV_BAD_POSITION = 0x10, 0x20, 0x40
+SQ_DEV_TIMEOUT, SQ_DEV_NONFINITE_LOGIT, SQ_DEV_BAD_POSITION, SQ_DEV_BAD_TOKEN_ID = 0x10, 0x20, 0x40, 0x80
 
 _P = ctypes.c_void_p
 _I64 = ctypes.c_int64
@@ -74,6 +75,9 @@ _SIGS = {
     "sq_attention": (_INT, [_P, _INT, _INT, _INT, _INT, _INT, _P, ctypes.c_float, _P, _P, _I64, _P, _P,
                             _SIZE, _P]),
     "sq_kv_rollback": (_INT, [_P, _P, _INT, _INT, _P, _P]),
+    "sq_embed": (_INT, [_P, _INT, _I64, _P, _I64, _I64, _P, _P]),
+    "sq_spec_commit": (_INT, [_P, _P, _INT, _INT, _INT, _P, _INT, _P, _P, _P, _P]),
+    "sq_spec_drafts": (_INT, [_P, _P, _INT, _INT, _P, _P, _P]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGS)
 
@@ -263,6 +267,36 @@ def sq_attention(qkv, B, T, Hq, Hkv, pos0, theta, k_cache, v_cache, out, workspa
 def sq_kv_rollback(base, n_accepted, limit, length, stream=None) -> None:
     _check("sq_kv_rollback", load().sq_kv_rollback(_ptr(base), _ptr(n_accepted), base.numel(), limit,
                                                    _ptr(length), _stream(stream)))
+
+
+def sq_embed(ids, table, out, stream=None, ids_stride: int = 1, M: int | None = None) -> None:
+    """out[m] = table[ids[m * ids_stride]] for m < M (default ids.numel());
+    ids int32, table fp16 [V, H], out fp16 [M, H]."""
+    V, H = table.shape
+    if M is None:
+        M = ids.numel()
+    _check("sq_embed", load().sq_embed(_ptr(ids), M, ids_stride, _ptr(table), V, H, _ptr(out),
+                                       _stream(stream)))
+
+
+def sq_spec_commit(n_accepted, tokens, hist, length, pos, last2, K: int, stream=None) -> None:
+    """Append each sequence's n_accepted[b] + 1 committed tokens (tokens int32
+    [B, ldt]; n_accepted None = one token) to hist int32 [B, cap] and
+    length [B]; write the next cycle's positions pos int32 [K + 1, B] and
+    the last two tokens last2 int32 [B, 2]."""
+    B, cap = hist.shape
+    ldt = tokens.shape[-1] if tokens.dim() > 1 else 1
+    _check("sq_spec_commit", load().sq_spec_commit(_ptr(n_accepted), _ptr(tokens), ldt, B, K, _ptr(hist),
+                                                   cap, _ptr(length), _ptr(pos), _ptr(last2),
+                                                   _stream(stream)))
+
+
+def sq_spec_drafts(samples, last2, verify_tokens, draft, stream=None) -> None:
+    """verify_tokens [B, K+1] = (last token, drafts), draft [B, K] =
+    samples^T from the draft steps' tokens samples int32 [K, B]."""
+    B, K1 = verify_tokens.shape
+    _check("sq_spec_drafts", load().sq_spec_drafts(_ptr(samples), _ptr(last2), B, K1 - 1,
+                                                   _ptr(verify_tokens), _ptr(draft), _stream(stream)))
 
 
 def sq_accept_workspace_bytes(B: int, K: int, V: int) -> int:

@@ -24,7 +24,7 @@
 // arithmetic (G * T * 2 D flops per cached key).
 #include <math.h>
 
-#include "sq_internal.h"
+#include "sq_decoder.h"
 
 namespace sq {
 
@@ -279,6 +279,105 @@ __global__ void __launch_bounds__(kHeadDim) attention_combine_kernel(const AttnA
   const int64_t row = (int64_t)b * a.T + t;
   a.out[row * (int64_t)a.Hq * kHeadDim + (int64_t)(kvh * a.G + g) * kHeadDim + d] =
       __float2half_rn(L > 0.0f ? O / L : 0.0f);
+}
+
+// ---- embedding ---------------------------------------------------------------------
+// out[m, :] = table[ids[m], :] (fp16 copy, 16-byte pieces when aligned); an id
+// outside [0, V) gives a zero row and sets SQ_DEV_BAD_TOKEN_ID.
+__global__ void __launch_bounds__(256) embed_kernel(const int32_t* __restrict__ ids, int64_t ids_stride,
+                                                    const __half* __restrict__ table, int64_t V,
+                                                    int64_t H, __half* __restrict__ out) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int64_t m = blockIdx.x;
+  const int32_t id = ids[m * ids_stride];
+  const bool ok = id >= 0 && (int64_t)id < V;
+  if (!ok && threadIdx.x == 0) atomicOr(&g_attn_status, SQ_DEV_BAD_TOKEN_ID);
+  const __half* src = table + (ok ? (int64_t)id : 0) * H;
+  __half* dst = out + m * H;
+  if ((H & 7) == 0 && ((reinterpret_cast<uintptr_t>(table) | reinterpret_cast<uintptr_t>(out)) & 15) == 0) {
+    for (int64_t i = threadIdx.x; i < H / 8; i += blockDim.x)
+      reinterpret_cast<uint4*>(dst)[i] = ok ? reinterpret_cast<const uint4*>(src)[i] : make_uint4(0, 0, 0, 0);
+  } else {
+    for (int64_t i = threadIdx.x; i < H; i += blockDim.x) dst[i] = ok ? src[i] : __ushort_as_half(0);
+  }
+}
+
+cudaError_t launch_embed(const int32_t* ids, int M, int64_t ids_stride, const __half* table, int64_t V,
+                         int64_t H, __half* out, cudaStream_t st) {
+  if (M == 0) return cudaSuccess;
+  return launch_pdl(embed_kernel, dim3((unsigned)M), dim3(256), 0, st, ids, ids_stride, table, V, H, out);
+}
+
+// ---- speculative bookkeeping (Sec. III-D.4: the accepted prefix plus the
+// correction becomes the context of the next cycle) ----------------------------------
+// One thread per sequence.  Appends the n + 1 committed tokens to the history
+// and derives the next cycle's inputs: the positions of the K draft steps and
+// of the verify pass, and the last two committed tokens (the draft's first
+// step re-reads the second-last one, whose key/value the draft may not have
+// computed when every draft was accepted).
+__global__ void spec_commit_kernel(const int32_t* __restrict__ n_acc, const int32_t* __restrict__ tokens,
+                                   int ldt, int B, int K, int32_t* __restrict__ hist, int cap,
+                                   int32_t* __restrict__ len, int32_t* __restrict__ pos,
+                                   int32_t* __restrict__ last2) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  int L = len[b];
+  int32_t* h = hist + (int64_t)b * cap;
+  bool bad = L < 0 || L > cap;
+  if (!bad) {
+    const int na = n_acc ? n_acc[b] : 0;
+    if (na >= ldt) {
+      bad = true;
+    } else if (na >= 0) {
+      const int cnt = na + 1 < cap - L ? na + 1 : cap - L;
+      for (int i = 0; i < cnt; ++i) h[L + i] = tokens[(int64_t)b * ldt + i];
+      if (cnt < na + 1) bad = true;
+      L += cnt;
+    }
+  }
+  if (bad || L < 2) {
+    atomicOr(&g_attn_status, SQ_DEV_BAD_POSITION);
+    if (L < 0 || L > cap) L = 0;
+  }
+  len[b] = L;
+  last2[2 * b] = L >= 2 ? h[L - 2] : -1;
+  last2[2 * b + 1] = L >= 1 ? h[L - 1] : -1;
+  if (K >= 1) pos[b] = L - 2;
+  for (int k = 1; k < K; ++k) pos[(int64_t)k * B + b] = L - 1 + k;
+  pos[(int64_t)K * B + b] = L - 1;
+}
+
+// verify_tokens[b, :] = (last committed token, draft 1 .. K); draft[b, k] =
+// samples[k, b] (the draft steps write one token per sequence).
+__global__ void spec_drafts_kernel(const int32_t* __restrict__ samples, const int32_t* __restrict__ last2,
+                                   int B, int K, int32_t* __restrict__ verify, int32_t* __restrict__ draft) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  verify[(int64_t)b * (K + 1)] = last2[2 * b + 1];
+  for (int k = 0; k < K; ++k) {
+    const int32_t t = samples[(int64_t)k * B + b];
+    verify[(int64_t)b * (K + 1) + 1 + k] = t;
+    draft[(int64_t)b * K + k] = t;
+  }
+}
+
+cudaError_t launch_spec_commit(const int32_t* n, const int32_t* tokens, int ldt, int B, int K, int32_t* hist,
+                               int cap, int32_t* len, int32_t* pos, int32_t* last2, cudaStream_t st) {
+  if (B == 0) return cudaSuccess;
+  return launch_pdl(spec_commit_kernel, dim3((unsigned)((B + 127) / 128)), dim3(128), 0, st, n, tokens, ldt,
+                    B, K, hist, cap, len, pos, last2);
+}
+
+cudaError_t launch_spec_drafts(const int32_t* samples, const int32_t* last2, int B, int K, int32_t* verify,
+                               int32_t* draft, cudaStream_t st) {
+  if (B == 0) return cudaSuccess;
+  return launch_pdl(spec_drafts_kernel, dim3((unsigned)((B + 127) / 128)), dim3(128), 0, st, samples, last2,
+                    B, K, verify, draft);
 }
 
 // ---- rollback -------------------------------------------------------------------

@@ -8,6 +8,7 @@
 #include <cmath>
 #include <string>
 
+#include "sq_decoder.h"
 #include "sq_internal.h"
 
 namespace sq {
@@ -480,6 +481,48 @@ sq_status sq_kv_rollback(const int32_t* base, const int32_t* n_accepted, int B, 
     return fail(SQ_ERR_ALIGN, "sq_kv_rollback: pointers must be 4-byte aligned");
   cudaError_t e = launch_kv_rollback(base, n_accepted, B, limit, len, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "sq_kv_rollback: launch");
+  return SQ_OK;
+}
+
+sq_status sq_embed(const int32_t* ids, int M, int64_t ids_stride, const void* table, int64_t V, int64_t H,
+                   void* out, sq_stream_t stream) {
+  if (M < 0 || V < 1 || H < 1 || ids_stride < 1)
+    return fail(SQ_ERR_SHAPE, "sq_embed: need M >= 0, V >= 1, H >= 1, ids_stride >= 1");
+  if (M == 0) return SQ_OK;
+  if (!ids || !table || !out) return fail(SQ_ERR_INVALID_ARG, "sq_embed: NULL pointer");
+  if (!aligned(ids, 4) || !aligned(table, 2) || !aligned(out, 2))
+    return fail(SQ_ERR_ALIGN, "sq_embed: misaligned pointer");
+  cudaError_t e = launch_embed(ids, M, ids_stride, reinterpret_cast<const __half*>(table), V, H,
+                               reinterpret_cast<__half*>(out), (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_embed: launch");
+  return SQ_OK;
+}
+
+sq_status sq_spec_commit(const int32_t* n_accepted, const int32_t* tokens, int ldt, int B, int K, int32_t* hist,
+                         int cap, int32_t* len, int32_t* pos, int32_t* last2, sq_stream_t stream) {
+  if (B < 0 || K < 0 || ldt < 1 || cap < 1)
+    return fail(SQ_ERR_SHAPE, "sq_spec_commit: need B >= 0, K >= 0, ldt >= 1, cap >= 1");
+  if (B == 0) return SQ_OK;
+  if (!tokens || !hist || !len || !pos || !last2) return fail(SQ_ERR_INVALID_ARG, "sq_spec_commit: NULL pointer");
+  if (!aligned(n_accepted, 4) || !aligned(tokens, 4) || !aligned(hist, 4) || !aligned(len, 4) ||
+      !aligned(pos, 4) || !aligned(last2, 4))
+    return fail(SQ_ERR_ALIGN, "sq_spec_commit: pointers must be 4-byte aligned");
+  cudaError_t e = launch_spec_commit(n_accepted, tokens, ldt, B, K, hist, cap, len, pos, last2,
+                                     (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_spec_commit: launch");
+  return SQ_OK;
+}
+
+sq_status sq_spec_drafts(const int32_t* samples, const int32_t* last2, int B, int K, int32_t* verify_tokens,
+                         int32_t* draft, sq_stream_t stream) {
+  if (B < 0 || K < 0) return fail(SQ_ERR_SHAPE, "sq_spec_drafts: need B >= 0, K >= 0");
+  if (B == 0) return SQ_OK;
+  if (!last2 || !verify_tokens || (K > 0 && (!samples || !draft)))
+    return fail(SQ_ERR_INVALID_ARG, "sq_spec_drafts: NULL pointer");
+  if (!aligned(samples, 4) || !aligned(last2, 4) || !aligned(verify_tokens, 4) || !aligned(draft, 4))
+    return fail(SQ_ERR_ALIGN, "sq_spec_drafts: pointers must be 4-byte aligned");
+  cudaError_t e = launch_spec_drafts(samples, last2, B, K, verify_tokens, draft, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_spec_drafts: launch");
   return SQ_OK;
 }
 

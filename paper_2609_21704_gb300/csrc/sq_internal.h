@@ -137,19 +137,4 @@ cudaError_t launch_accept_logits(const AcceptArgs& a, const SoftmaxArgs& sa, cud
 cudaError_t launch_softmax(const SoftmaxArgs& sa, float* p, cudaStream_t st);
 cudaError_t take_accept_status(uint32_t* bits);
 
-// sq_attention.cu: RMSNorm, RoPE + KV append, decode attention, rollback
-cudaError_t launch_rmsnorm(const __half* x, const __half* gamma, int M, int64_t H, float eps, __half* y,
-                           cudaStream_t st);
-cudaError_t launch_kv_append(const __half* qkv, int B, int T, int Hq, int Hkv, const int32_t* pos0,
-                             double theta, __half* kc, __half* vc, int64_t max_ctx, cudaStream_t st);
-size_t attention_workspace_bytes(int B, int T, int Hq, int Hkv, int64_t max_ctx);
-size_t attention_smem_bytes(int Q);
-int attention_max_tokens();  // T limit of sq_kv_append / sq_attention
-cudaError_t launch_attention(const __half* qkv, int B, int T, int Hq, int Hkv, const int32_t* pos0,
-                             double theta, const __half* kc, const __half* vc, int64_t max_ctx,
-                             __half* out, void* ws, cudaStream_t st);
-cudaError_t launch_kv_rollback(const int32_t* base, const int32_t* n, int B, int limit, int32_t* len,
-                               cudaStream_t st);
-cudaError_t take_attn_status(uint32_t* bits);
-
 }  // namespace sq

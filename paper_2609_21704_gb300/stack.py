@@ -67,10 +67,13 @@ class LinearStack:
     and the requested derived variants, resident on ``device``."""
 
     def __init__(self, shape: StackShape, device, seed: int = 0, variants=("int4", "fp8"),
-                 layers: int | None = None, with_lm_head: bool = True):
+                 layers: int | None = None, with_lm_head: bool = True, host_weights: bool = False):
         self.shape = shape
         self.device = torch.device(device)
         self.variants = tuple(variants)
+        # host_weights: draw the parents with numpy on the host (small test
+        # models whose weights the oracle regenerates from the same seeds)
+        self.host_weights = host_weights
         self.layers = []
         nl = shape.layers if layers is None else layers
         s = seed
@@ -85,9 +88,29 @@ class LinearStack:
         if with_lm_head:
             name, n, k = shape.lm_head()
             self.lm_head = self._make(name, n, k, SQ_EPI_NONE, s)
+            s += 1
+        self._embed_seed = s
+        self._embed = None
+
+    def embedding(self) -> torch.Tensor:
+        """The input embedding, fp16 [vocab, hidden]: its own seeded table
+        (untied from the lm_head), drawn on first use and shared by the
+        parent and its variants (only the linear layers are quantised)."""
+        if self._embed is None:
+            sh = self.shape
+            ws = synth.stack_weight_seed(self._embed_seed, 0)
+            if self.host_weights:
+                self._embed = torch.from_numpy(synth.weights_fp16(ws, sh.vocab, sh.hidden)).to(self.device)
+            else:
+                self._embed = synth.weights_fp16_device(ws, sh.vocab, sh.hidden, self.device)
+        return self._embed
 
     def _make(self, name, n, k, epi, seed) -> Proj:
-        w16 = synth.weights_fp16_device(seed * 7919 + 17, n, k, self.device)
+        ws = synth.stack_weight_seed(seed, 0)
+        if self.host_weights:
+            w16 = torch.from_numpy(synth.weights_fp16(ws, n, k)).to(self.device)
+        else:
+            w16 = synth.weights_fp16_device(ws, n, k, self.device)
         q = {}
         for v in self.variants:
             kind = SQ_INT4_G128 if v == "int4" else SQ_FP8_E4M3_ROW
@@ -180,20 +203,29 @@ class DecoderState:
     """Per-model state of a decoder pass over T new tokens of B sequences: a
     KV cache per layer ([B, Hkv, max_ctx, 128] fp16, keys rotated), the
     RMSNorm gains, the residual stream and the pass's activations.  Token t
-    of sequence b sits at position pos0[b] + t."""
+    of sequence b sits at position pos0[b] + t.  `share` gives another
+    state whose caches and gains this one uses (states of one model at
+    different T); `share_gains` gives only the gains (a second model)."""
 
-    def __init__(self, stack: LinearStack, B: int, T: int, max_ctx: int, context: int,
-                 seed: int = 5):
+    def __init__(self, stack: LinearStack, B: int, T: int, max_ctx: int, context: int = 0,
+                 seed: int = 5, share: "DecoderState | None" = None,
+                 share_gains: "DecoderState | None" = None):
         from . import sq_attention_workspace_bytes
         sh, dev = stack.shape, stack.device
         self.B, self.T, self.max_ctx = B, T, max_ctx
         nl = len(stack.layers)
-        cache = (B, sh.kv_heads, max_ctx, HEAD_DIM)
-        self.k = [torch.zeros(cache, dtype=torch.float16, device=dev) for _ in range(nl)]
-        self.v = [torch.zeros(cache, dtype=torch.float16, device=dev) for _ in range(nl)]
-        g = [1.0 + synth.fp16_normal(seed + i, (sh.hidden,), 0.05).astype("float32")
-             for i in range(2 * nl + 1)]
-        self.gamma = [torch.from_numpy(a.astype("float16")).to(dev) for a in g]
+        if share is not None:
+            assert share.B == B and share.max_ctx == max_ctx
+            self.k, self.v = share.k, share.v
+        else:
+            cache = (B, sh.kv_heads, max_ctx, HEAD_DIM)
+            self.k = [torch.zeros(cache, dtype=torch.float16, device=dev) for _ in range(nl)]
+            self.v = [torch.zeros(cache, dtype=torch.float16, device=dev) for _ in range(nl)]
+        src = share if share is not None else share_gains
+        if src is not None:
+            self.gamma = src.gamma
+        else:
+            self.gamma = [torch.from_numpy(g).to(dev) for g in synth.rms_gains(seed, sh.hidden, 2 * nl + 1)]
         self.pos0 = torch.full((B,), context, dtype=torch.int32, device=dev)
         M = B * T
         self.x = synth.activations_fp16_device(seed + 99, M, sh.hidden, dev)
@@ -203,28 +235,34 @@ class DecoderState:
         self.g = torch.empty((M, sh.intermediate), dtype=torch.float16, device=dev)
         self.logits = torch.empty((M, sh.vocab), dtype=torch.float16, device=dev) \
             if stack.lm_head is not None else None
+        # the last token of each sequence, for passes whose lm_head reads only it
+        self.last_rows = torch.arange(B, dtype=torch.int32, device=dev) * T + (T - 1)
+        self.x_last = torch.empty((B, sh.hidden), dtype=torch.float16, device=dev)
         self.ws = torch.empty(sq_attention_workspace_bytes(B, T, sh.q_heads, sh.kv_heads, max_ctx),
                               dtype=torch.uint8, device=dev)
 
 
 def decoder_pass(stack: LinearStack, variant: str, st: DecoderState, stream=None,
-                 logits=None) -> None:
+                 logits=None, pos0=None, last_only: bool = False, with_logits: bool = True) -> None:
     """One decoder step (draft or verify) with the variant's weights: per
     layer x += o(attn(rope(qkv(norm(x))))), x += down(silu-gate(norm(x)));
     then logits = lm_head(norm(x)) (into `logits` when given).  The new
     tokens' keys and values are appended to the caches before attention
-    reads them."""
-    from . import SQ_EPI_RESIDUAL, sq_attention, sq_kv_append, sq_rmsnorm
+    reads them.  pos0 (int32 [B], device) overrides st.pos0; last_only
+    runs the lm_head on each sequence's last token only (logits [B, V]);
+    with_logits=False stops after the layers (a prefill that only fills
+    the cache)."""
+    from . import SQ_EPI_RESIDUAL, sq_attention, sq_embed, sq_kv_append, sq_rmsnorm
     sh = stack.shape
     wk = WKIND[variant]
     B, T = st.B, st.T
+    pos = st.pos0 if pos0 is None else pos0
     for li, (qkv, o, gu, down) in enumerate(stack.layers):
         sq_rmsnorm(st.x, st.gamma[2 * li], RMS_EPS, st.h, stream)
         w, s = qkv.weight(variant)
         sq_linear_ex(wk, st.h, w, s, None, None, SQ_EPI_NONE, st.qkv, stream)
-        sq_kv_append(st.qkv, B, T, sh.q_heads, sh.kv_heads, st.pos0, ROPE_THETA, st.k[li], st.v[li],
-                     stream)
-        sq_attention(st.qkv, B, T, sh.q_heads, sh.kv_heads, st.pos0, ROPE_THETA, st.k[li], st.v[li],
+        sq_kv_append(st.qkv, B, T, sh.q_heads, sh.kv_heads, pos, ROPE_THETA, st.k[li], st.v[li], stream)
+        sq_attention(st.qkv, B, T, sh.q_heads, sh.kv_heads, pos, ROPE_THETA, st.k[li], st.v[li],
                      st.attn, st.ws, stream)
         w, s = o.weight(variant)
         sq_linear_ex(wk, st.attn, w, s, None, st.x, SQ_EPI_RESIDUAL, st.x, stream)
@@ -233,8 +271,12 @@ def decoder_pass(stack: LinearStack, variant: str, st: DecoderState, stream=None
         sq_linear_ex(wk, st.h, w, s, None, None, SQ_EPI_SILU_GATE, st.g, stream)
         w, s = down.weight(variant)
         sq_linear_ex(wk, st.g, w, s, None, st.x, SQ_EPI_RESIDUAL, st.x, stream)
-    if stack.lm_head is not None:
-        sq_rmsnorm(st.x, st.gamma[-1], RMS_EPS, st.h, stream)
-        w, s = stack.lm_head.weight(variant)
-        sq_linear_ex(wk, st.h, w, s, None, None, SQ_EPI_NONE, st.logits if logits is None else logits,
-                     stream)
+    if stack.lm_head is None or not with_logits:
+        return
+    x, h = st.x, st.h
+    if last_only and T > 1:
+        sq_embed(st.last_rows, st.x, st.x_last, stream)   # row gather
+        x, h = st.x_last, st.h[:B]
+    sq_rmsnorm(x, st.gamma[-1], RMS_EPS, h, stream)
+    w, s = stack.lm_head.weight(variant)
+    sq_linear_ex(wk, h, w, s, None, None, SQ_EPI_NONE, st.logits if logits is None else logits, stream)

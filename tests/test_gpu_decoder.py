@@ -97,3 +97,20 @@ def test_append_outside_the_cache_sets_status():
     vc = torch.zeros_like(kc)
     sq.sq_kv_append(qkv, B, T, Hq, Hkv, _t(np.array([62], np.int32)), THETA, kc, vc)
     assert sq.sq_check() & sq.SQ_DEV_BAD_POSITION
+
+
+def test_embed_gathers_rows_exactly():
+    rng = np.random.default_rng(11)
+    V, H = 1000, 1536
+    table = rng.normal(0, 1, (V, H)).astype(np.float16)
+    ids = np.array([0, 999, 17, 17, 500], np.int32)
+    out = torch.empty(len(ids), H, dtype=torch.float16, device=dev())
+    sq.sq_embed(_t(ids), _t(table), out)
+    assert sq.sq_check() == 0
+    assert np.array_equal(out.cpu().numpy().view(np.uint16), table[ids].view(np.uint16))
+    bad = _t(np.array([5, 1000], np.int32))
+    out2 = torch.empty(2, H, dtype=torch.float16, device=dev())
+    sq.sq_embed(bad, _t(table), out2)
+    assert sq.sq_check() & sq.SQ_DEV_BAD_TOKEN_ID
+    assert np.array_equal(out2[0].cpu().numpy().view(np.uint16), table[5].view(np.uint16))
+    assert bool((out2[1] == 0).all())
