@@ -83,6 +83,7 @@ class Generator:
         self.verify_in = torch.zeros((B, K + 1), **i32)
         self.draft_tok = torch.zeros((B, kk), **i32)
         self.n = torch.zeros((B,), **i32)
+        self.n_pick = torch.zeros((B,), **i32)      # the greedy pick's (unused) accepted count
         self.tok = torch.zeros((B, K + 1), **i32)
         self.tok1 = torch.zeros((B, 1), **i32)
         self.zq = torch.empty((kk, B, V), dtype=torch.float16, device=dev)
@@ -101,7 +102,7 @@ class Generator:
         """One token per sequence from fp16 logits z [B, V] into out (int32, B)."""
         if self.mode == SQ_ACCEPT_GREEDY:
             sq_accept_logits(z.view(self.B, 1, -1), None, None, u, self.temperature, SQ_ACCEPT_GREEDY,
-                             None, out, self.ws_pick, stream)
+                             self.n_pick, out, self.ws_pick, stream)
         else:
             sq_sample_logits(z, u, self.temperature, out, self.ws_pick, stream)
 
