@@ -447,7 +447,9 @@ def main():
         del g_pf16, g_pfd, bp
 
         # the decoder step around the stack (RMSNorm, RoPE, KV cache,
-        # grouped-query attention) at a 1000-token context: each pass alone,
+        # grouped-query attention) at a 1000-token context, RMSNorm fused
+        # into the projections and the append into the attention (the draft
+        # pass also unfused, for comparison): each pass alone,
         # a whole speculative cycle on decoder passes (drafts write their
         # logits slot and sample, verify, accept, cache rollback) and direct
         # decoding with the FP16 parent
@@ -469,6 +471,9 @@ def main():
             stk.decoder_pass(stack, "fp16", dd, stream, logits=zq[0])
             sq.sq_sample_logits(zq[0], u_draft[0], temperature, samp[0], ws_s, stream)
 
+        g_ddu = capture(lambda: stk.decoder_pass(stack, args.draft, dd, stream, fused=False))
+        t_ddu = timed(g_ddu, reps) / reps
+        del g_ddu
         g_dd = capture(lambda: stk.decoder_pass(stack, args.draft, dd, stream))
         g_dv = capture(lambda: stk.decoder_pass(stack, "fp16", dv, stream))
         g_dc = capture(dec_cycle)
@@ -643,6 +648,7 @@ def main():
             "speedup_vs_direct_fp16": value / (B * world / t_direct),
             "decoder_context": ctx,
             "decoder_draft_pass_ms": 1e3 * t_dd,
+            "decoder_draft_pass_unfused_ms": 1e3 * t_ddu,
             "decoder_verify_pass_ms": 1e3 * t_dv,
             "decoder_cycle_ms": 1e3 * t_dc,
             "decoder_tokens_per_s": B * world * mean_tokens / t_dc,

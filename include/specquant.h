@@ -158,6 +158,18 @@ SQ_API sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, cons
                        const void* bias, const void* residual, sq_epilogue epi, void* y,
                        int M, int64_t N, int64_t K, sq_stream_t stream);
 
+/* sq_linear_norm: y = epi((rmsnorm(x) * gamma) W'^T + bias) -- the decoder's
+ * pre-norm projections (q/k/v, gate/up, lm_head) in one call.  rmsnorm is
+ * sq_rmsnorm's (fp32 arithmetic, the normalised rows rounded to fp16) and
+ * the result is bit-identical to sq_rmsnorm followed by sq_linear_ex.  The
+ * CUDA-core GEMV normalises the activation rows as it stages them (no extra
+ * launch); the tensor-core path writes them to xn (fp16 [M, K], 16-byte
+ * aligned, not aliasing x, y or the residual) first.  gamma fp16 [K], 16-byte
+ * aligned; eps >= 0. */
+SQ_API sq_status sq_linear_norm(sq_wkind wkind, const void* x, const void* gamma, float eps, void* xn,
+                                const void* w, const void* scales, const void* bias, const void* residual,
+                                sq_epilogue epi, void* y, int M, int64_t N, int64_t K, sq_stream_t stream);
+
 /* Engine sq_linear_ex would use for these sizes: 1 = tcgen05 tensor cores,
  * 0 = CUDA-core GEMV, -1 = sizes or kinds sq_linear_ex rejects (pointers are
  * not examined; nothing runs on the device).  The paper has no counterpart:
@@ -327,6 +339,16 @@ SQ_API sq_status sq_attention(const void* qkv, int B, int T, int Hq, int Hkv, in
                               const int32_t* pos0, float theta, const void* k_cache,
                               const void* v_cache, int64_t max_ctx, void* out, void* workspace,
                               size_t ws_bytes, sq_stream_t stream);
+/* sq_attention_append: sq_kv_append followed by sq_attention in one launch
+ * (same arguments; the caches are written): the cache chunk that holds a
+ * new token's position rotates its key from qkv, writes key and value, and
+ * attends to them directly.  Caches and output are bit-identical to the two
+ * calls.  A position outside [0, max_ctx) writes nothing, sets
+ * SQ_DEV_BAD_POSITION and leaves the sequence's output rows zero. */
+SQ_API sq_status sq_attention_append(const void* qkv, int B, int T, int Hq, int Hkv, int D,
+                                     const int32_t* pos0, float theta, void* k_cache, void* v_cache,
+                                     int64_t max_ctx, void* out, void* workspace, size_t ws_bytes,
+                                     sq_stream_t stream);
 SQ_API sq_status sq_kv_rollback(const int32_t* base, const int32_t* n_accepted, int B, int limit,
                                 int32_t* len, sq_stream_t stream);
 /* sq_embed: out[m, :] = table[ids[m * ids_stride], :] for M token ids

@@ -30,7 +30,7 @@ __all__ = [
     "sq_accept_logits_workspace_bytes", "sq_accept_logits", "sq_sample_logits",
     "sq_softmax_workspace_bytes", "sq_softmax", "sq_rmsnorm", "sq_kv_append",
     "sq_attention_workspace_bytes", "sq_attention", "sq_kv_rollback", "sq_embed",
-    "sq_spec_commit", "sq_spec_drafts",
+    "sq_attention_append", "sq_linear_norm", "sq_spec_commit", "sq_spec_drafts",
     "EXPORTED_SYMBOLS",
 ]
 
@@ -57,6 +57,8 @@ _SIGS = {
     "sq_linear_fp8": (_INT, [_P, _P, _P, _P, _P, _INT, _I64, _I64, _P]),
     "sq_verify": (_INT, [_P, _P, _P, _P, _INT, _I64, _I64, _P]),
     "sq_linear_ex": (_INT, [_INT, _P, _P, _P, _P, _P, _INT, _P, _INT, _I64, _I64, _P]),
+    "sq_linear_norm": (_INT, [_INT, _P, _P, ctypes.c_float, _P, _P, _P, _P, _P, _INT, _P, _INT, _I64,
+                              _I64, _P]),
     "sq_accept_workspace_bytes": (_SIZE, [_INT, _INT, _I64]),
     "sq_accept": (_INT, [_P, _P, _P, _P, _INT, _INT, _I64, _INT, _P, _P, _P, _SIZE, _P]),
     "sq_sample": (_INT, [_P, _P, _INT, _I64, _P, _P, _SIZE, _P]),
@@ -76,6 +78,8 @@ _SIGS = {
                             _SIZE, _P]),
     "sq_kv_rollback": (_INT, [_P, _P, _INT, _INT, _P, _P]),
     "sq_embed": (_INT, [_P, _INT, _I64, _P, _I64, _I64, _P, _P]),
+    "sq_attention_append": (_INT, [_P, _INT, _INT, _INT, _INT, _INT, _P, ctypes.c_float, _P, _P, _I64, _P,
+                                   _P, _SIZE, _P]),
     "sq_spec_commit": (_INT, [_P, _P, _INT, _INT, _INT, _P, _INT, _P, _P, _P, _P]),
     "sq_spec_drafts": (_INT, [_P, _P, _INT, _INT, _P, _P, _P]),
 }
@@ -163,6 +167,16 @@ def sq_linear_ex(wkind, x, w, scales, bias, residual, epi, y, stream=None) -> No
     _check("sq_linear_ex", load().sq_linear_ex(wkind, _ptr(x), _ptr(w), _ptr(scales), _ptr(bias),
                                                _ptr(residual), epi, _ptr(y), M, N, K,
                                                _stream(stream)))
+
+
+def sq_linear_norm(wkind, x, gamma, eps, xn, w, scales, bias, residual, epi, y, stream=None) -> None:
+    """y = linear(rmsnorm(x) * gamma); xn fp16 [M, K] scratch for the
+    normalised rows (written only where the engine needs them in memory)."""
+    M, K = x.shape
+    N = y.shape[1]
+    _check("sq_linear_norm", load().sq_linear_norm(wkind, _ptr(x), _ptr(gamma), float(eps), _ptr(xn), _ptr(w),
+                                                   _ptr(scales), _ptr(bias), _ptr(residual), epi, _ptr(y),
+                                                   M, N, K, _stream(stream)))
 
 
 class SqLinearOp(ctypes.Structure):
@@ -259,6 +273,15 @@ def sq_attention(qkv, B, T, Hq, Hkv, pos0, theta, k_cache, v_cache, out, workspa
                  stream=None) -> None:
     """out fp16 [B*T, Hq*128] = causal GQA attention of the new tokens over the caches."""
     _check("sq_attention", load().sq_attention(
+        _ptr(qkv), B, T, Hq, Hkv, 128, _ptr(pos0), float(theta), _ptr(k_cache), _ptr(v_cache),
+        k_cache.shape[2], _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
+        _stream(stream)))
+
+
+def sq_attention_append(qkv, B, T, Hq, Hkv, pos0, theta, k_cache, v_cache, out, workspace,
+                        stream=None) -> None:
+    """sq_kv_append + sq_attention in one launch (the caches are written)."""
+    _check("sq_attention_append", load().sq_attention_append(
         _ptr(qkv), B, T, Hq, Hkv, 128, _ptr(pos0), float(theta), _ptr(k_cache), _ptr(v_cache),
         k_cache.shape[2], _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
         _stream(stream)))

@@ -83,6 +83,15 @@ __device__ __forceinline__ float2 rope_cs(int pos, double f) {
   return make_float2(c, s);
 }
 
+// The rotated pair (x1 c - x2 s, x2 c + x1 s), rounded to fp16 as the cache
+// stores it; the products and differences are rounded one by one (no
+// contraction), so the separate append and the fused attention write the
+// same bits.
+__device__ __forceinline__ void rope_rotate_f16(float x1, float x2, float2 cs, __half& y1, __half& y2) {
+  y1 = __float2half_rn(__fsub_rn(__fmul_rn(x1, cs.x), __fmul_rn(x2, cs.y)));
+  y2 = __float2half_rn(__fadd_rn(__fmul_rn(x2, cs.x), __fmul_rn(x1, cs.y)));
+}
+
 // One CTA per (token row, key/value head): rotate the new key, copy the
 // value, both into the caches at the token's position.
 __global__ void __launch_bounds__(64) kv_append_kernel(const __half* __restrict__ qkv, int T, int Hq,
@@ -104,10 +113,8 @@ __global__ void __launch_bounds__(64) kv_append_kernel(const __half* __restrict_
   const int64_t dst = (((int64_t)b * Hkv + h) * max_ctx + pos) * kHeadDim;
   const int d = threadIdx.x;  // pair (d, d + D/2)
   const float2 cs = rope_cs(pos, rf.f[d]);
-  const float c = cs.x, s = cs.y;
-  const float x1 = __half2float(kr[d]), x2 = __half2float(kr[d + kHeadDim / 2]);
-  kc[dst + d] = __float2half_rn(x1 * c - x2 * s);
-  kc[dst + d + kHeadDim / 2] = __float2half_rn(x2 * c + x1 * s);
+  rope_rotate_f16(__half2float(kr[d]), __half2float(kr[d + kHeadDim / 2]), cs, kc[dst + d],
+                  kc[dst + d + kHeadDim / 2]);
   vc[dst + d] = vr[d];
   vc[dst + d + kHeadDim / 2] = vr[d + kHeadDim / 2];
 }
@@ -117,6 +124,9 @@ struct AttnArgs {
   const __half* qkv;
   const __half* kc;
   const __half* vc;
+  __half* kcw;  // the same caches, written when append != 0
+  __half* vcw;
+  int append;   // the new tokens' keys/values are appended by the chunk that holds them
   const int32_t* pos0;
   __half* out;
   float* part;  // [(B*Hkv) * nsplit * Q * kPartStride]: per query (m, l, -, -, o[D])
@@ -147,6 +157,8 @@ __global__ void __launch_bounds__(kAttnThreads) attention_partial_kernel(const A
   const int64_t len = (int64_t)p0 + T;  // cache entries after the append
   const int64_t j0 = (int64_t)split * kAttnChunk;
   float* part = a.part + ((int64_t)bh * a.nsplit + split) * Q * kPartStride;
+  if (a.append && (p0 < 0 || len > a.max_ctx) && split == 0 && tid == 0)
+    atomicOr(&g_attn_status, SQ_DEV_BAD_POSITION);
   if (j0 >= len || p0 < 0 || len > a.max_ctx) {  // empty chunk: neutral partials
     for (int q = tid; q < Q; q += kAttnThreads) {
       part[(int64_t)q * kPartStride] = -INFINITY;
@@ -161,11 +173,36 @@ __global__ void __launch_bounds__(kAttnThreads) attention_partial_kernel(const A
     cst[idx] = rope_cs(p0 + t, a.rf.f[d]);
   }
   const int64_t cbase = (((int64_t)b * a.Hkv + kvh) * a.max_ctx + j0) * kHeadDim;
+  // positions p0 .. p0+T-1 are the new tokens: with append, this chunk's
+  // share of them is rotated from qkv, written to the caches and used
+  // directly (every position belongs to one chunk, so each is written once)
+  const int j_new = a.append ? (int)((int64_t)p0 - j0) : kAttnChunk;  // first new key of the chunk
+  if (j_new < nk) __syncthreads();  // cst is read below
   for (int idx = tid; idx < kAttnChunk * kHeadDim; idx += kAttnThreads) {
     const int j = idx / kHeadDim, d = idx - j * kHeadDim;
-    const bool in = j < nk;
-    ks[j * kRowPad + d] = in ? __half2float(a.kc[cbase + idx]) : 0.0f;
-    vs[j * kRowPad + d] = in ? __half2float(a.vc[cbase + idx]) : 0.0f;
+    float kf = 0.0f, vf = 0.0f;
+    if (j < nk) {
+      if (j >= j_new) {
+        const int t = (int)(j0 + j - p0);
+        const __half* row = a.qkv + ((int64_t)b * T + t) * width;
+        const __half* kr = row + (int64_t)(a.Hq + kvh) * kHeadDim;
+        const __half vh = row[(int64_t)(a.Hq + a.Hkv + kvh) * kHeadDim + d];
+        const int pd = d & (kHeadDim / 2 - 1);
+        __half y1, y2;
+        rope_rotate_f16(__half2float(kr[pd]), __half2float(kr[pd + kHeadDim / 2]),
+                        cst[t * (kHeadDim / 2) + pd], y1, y2);
+        const __half kh = d < kHeadDim / 2 ? y1 : y2;
+        a.kcw[cbase + idx] = kh;
+        a.vcw[cbase + idx] = vh;
+        kf = __half2float(kh);
+        vf = __half2float(vh);
+      } else {
+        kf = __half2float(a.kc[cbase + idx]);
+        vf = __half2float(a.vc[cbase + idx]);
+      }
+    }
+    ks[j * kRowPad + d] = kf;
+    vs[j * kRowPad + d] = vf;
   }
   __syncthreads();
   for (int idx = tid; idx < Q * (kHeadDim / 2); idx += kAttnThreads) {
@@ -427,12 +464,16 @@ int attention_max_tokens() { return kMaxT; }
 
 cudaError_t launch_attention(const __half* qkv, int B, int T, int Hq, int Hkv, const int32_t* pos0,
                              double theta, const __half* kc, const __half* vc, int64_t max_ctx,
-                             __half* out, void* ws, cudaStream_t st) {
+                             __half* out, void* ws, cudaStream_t st, __half* kc_append,
+                             __half* vc_append) {
   if (B == 0 || T == 0) return cudaSuccess;
   AttnArgs a = {};
   a.qkv = qkv;
   a.kc = kc;
   a.vc = vc;
+  a.kcw = kc_append;
+  a.vcw = vc_append;
+  a.append = kc_append != nullptr && vc_append != nullptr;
   a.pos0 = pos0;
   a.out = out;
   a.part = reinterpret_cast<float*>(ws);

@@ -153,9 +153,14 @@ static sq_status check_linear(const sq_linear_op& op) {
 }
 
 // Launches one checked call.
-static sq_status run_linear(const sq_linear_op& op, cudaStream_t stream) {
+// gamma != null: y = linear(rmsnorm(x) * gamma).  The GEMV normalises the rows
+// it stages; the tensor-core path writes the normalised rows to xn first.
+static sq_status run_linear(const sq_linear_op& op, cudaStream_t stream, const __half* gamma = nullptr,
+                            float eps = 0.0f, __half* xn = nullptr) {
   GemvArgs a = {};
   a.x = reinterpret_cast<const __half*>(op.x);
+  a.gamma = gamma;
+  a.eps = eps;
   a.w = reinterpret_cast<const uint8_t*>(op.w);
   a.scales = op.scales;
   a.bias = reinterpret_cast<const __half*>(op.bias);
@@ -171,6 +176,11 @@ static sq_status run_linear(const sq_linear_op& op, cudaStream_t stream) {
   cudaError_t e;
   if (use_tensor_cores(op.wkind, op.M, op.N, op.K, op.epi) && tc_supported(op.M, op.K, op.epi)) {
     // tcgen05 tensor cores, weights on the MMA's M side
+    if (gamma) {
+      e = launch_rmsnorm(a.x, gamma, op.M, op.K, eps, xn, stream);
+      if (e != cudaSuccess) return cuda_fail(e, "sq_linear_norm: rmsnorm launch");
+      a.x = xn;
+    }
     e = launch_tc(op.wkind, a.x, op.w, op.scales, a.bias, a.residual, a.y, op.M, op.N, op.K, op.epi,
                   stream);
     if (e != cudaSuccess) return cuda_fail(e, "sq_linear: tensor-core launch");
@@ -179,6 +189,34 @@ static sq_status run_linear(const sq_linear_op& op, cudaStream_t stream) {
   e = launch_gemv(op.wkind, a, stream);
   if (e != cudaSuccess) return cuda_fail(e, "sq_linear: launch");
   return SQ_OK;
+}
+
+sq_status sq_linear_norm(sq_wkind wkind, const void* x, const void* gamma, float eps, void* xn, const void* w,
+                         const void* scales, const void* bias, const void* residual, sq_epilogue epi, void* y,
+                         int M, int64_t N, int64_t K, sq_stream_t stream) {
+  sq_linear_op op = {};
+  op.wkind = wkind;
+  op.epi = epi;
+  op.M = M;
+  op.N = N;
+  op.K = K;
+  op.x = x;
+  op.w = w;
+  op.scales = scales;
+  op.bias = bias;
+  op.residual = residual;
+  op.y = y;
+  sq_status st = check_linear(op);
+  if (st != SQ_OK) return st;
+  if (M == 0 || N == 0) return SQ_OK;
+  if (!gamma || !xn) return fail(SQ_ERR_INVALID_ARG, "sq_linear_norm: NULL gamma or xn");
+  if (!aligned(gamma, 16) || !aligned(xn, 16))
+    return fail(SQ_ERR_ALIGN, "sq_linear_norm: gamma and xn must be 16-byte aligned");
+  if (!(eps >= 0.0f) || !std::isfinite(eps)) return fail(SQ_ERR_INVALID_ARG, "sq_linear_norm: bad eps");
+  if (xn == y || xn == x || (residual && xn == residual))
+    return fail(SQ_ERR_INVALID_ARG, "sq_linear_norm: xn must not alias x, y or the residual");
+  return run_linear(op, (cudaStream_t)stream, reinterpret_cast<const __half*>(gamma), eps,
+                    reinterpret_cast<__half*>(xn));
 }
 
 sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void* scales,
@@ -450,26 +488,43 @@ size_t sq_attention_workspace_bytes(int B, int T, int Hq, int Hkv, int D, int64_
   return attention_workspace_bytes(B, T, Hq, Hkv, max_ctx);
 }
 
-sq_status sq_attention(const void* qkv, int B, int T, int Hq, int Hkv, int D, const int32_t* pos0,
-                       float theta, const void* k_cache, const void* v_cache, int64_t max_ctx, void* out,
-                       void* workspace, size_t ws_bytes, sq_stream_t stream) {
-  sq_status st = check_attn("sq_attention", qkv, B, T, Hq, Hkv, D, pos0, theta, k_cache, v_cache, max_ctx);
+static sq_status attention_common(const char* who, const void* qkv, int B, int T, int Hq, int Hkv, int D,
+                                  const int32_t* pos0, float theta, const void* k_cache, const void* v_cache,
+                                  int64_t max_ctx, void* out, void* workspace, size_t ws_bytes, bool append,
+                                  sq_stream_t stream) {
+  sq_status st = check_attn(who, qkv, B, T, Hq, Hkv, D, pos0, theta, k_cache, v_cache, max_ctx);
   if (st != SQ_OK) return st;
   if (B == 0 || T == 0) return SQ_OK;
-  if (!out || !aligned(out, 2)) return fail(SQ_ERR_ALIGN, "sq_attention: out NULL or misaligned");
+  if (!out || !aligned(out, 2)) return fail(SQ_ERR_ALIGN, "%s: out NULL or misaligned", who);
   const size_t need = attention_workspace_bytes(B, T, Hq, Hkv, max_ctx);
   if (!workspace || ws_bytes < need)
-    return fail(SQ_ERR_WORKSPACE, "sq_attention: workspace %zu bytes < %zu required", ws_bytes, need);
-  if (!aligned(workspace, 16)) return fail(SQ_ERR_ALIGN, "sq_attention: workspace must be 16-byte aligned");
+    return fail(SQ_ERR_WORKSPACE, "%s: workspace %zu bytes < %zu required", who, ws_bytes, need);
+  if (!aligned(workspace, 16)) return fail(SQ_ERR_ALIGN, "%s: workspace must be 16-byte aligned", who);
   if (attention_smem_bytes((Hq / Hkv) * T) > (size_t)device_max_smem())
-    return fail(SQ_ERR_SHAPE, "sq_attention: query group too large for shared memory");
-  if (max_ctx > ((int64_t)1 << 17)) return fail(SQ_ERR_SHAPE, "sq_attention: max_ctx > 2^17");
+    return fail(SQ_ERR_SHAPE, "%s: query group too large for shared memory", who);
+  if (max_ctx > ((int64_t)1 << 17)) return fail(SQ_ERR_SHAPE, "%s: max_ctx > 2^17", who);
+  __half* kw = append ? reinterpret_cast<__half*>(const_cast<void*>(k_cache)) : nullptr;
+  __half* vw = append ? reinterpret_cast<__half*>(const_cast<void*>(v_cache)) : nullptr;
   cudaError_t e = launch_attention(reinterpret_cast<const __half*>(qkv), B, T, Hq, Hkv, pos0, (double)theta,
                                    reinterpret_cast<const __half*>(k_cache),
                                    reinterpret_cast<const __half*>(v_cache), max_ctx,
-                                   reinterpret_cast<__half*>(out), workspace, (cudaStream_t)stream);
-  if (e != cudaSuccess) return cuda_fail(e, "sq_attention: launch");
+                                   reinterpret_cast<__half*>(out), workspace, (cudaStream_t)stream, kw, vw);
+  if (e != cudaSuccess) return cuda_fail(e, who);
   return SQ_OK;
+}
+
+sq_status sq_attention(const void* qkv, int B, int T, int Hq, int Hkv, int D, const int32_t* pos0,
+                       float theta, const void* k_cache, const void* v_cache, int64_t max_ctx, void* out,
+                       void* workspace, size_t ws_bytes, sq_stream_t stream) {
+  return attention_common("sq_attention", qkv, B, T, Hq, Hkv, D, pos0, theta, k_cache, v_cache, max_ctx, out,
+                          workspace, ws_bytes, false, stream);
+}
+
+sq_status sq_attention_append(const void* qkv, int B, int T, int Hq, int Hkv, int D, const int32_t* pos0,
+                              float theta, void* k_cache, void* v_cache, int64_t max_ctx, void* out,
+                              void* workspace, size_t ws_bytes, sq_stream_t stream) {
+  return attention_common("sq_attention_append", qkv, B, T, Hq, Hkv, D, pos0, theta, k_cache, v_cache,
+                          max_ctx, out, workspace, ws_bytes, true, stream);
 }
 
 sq_status sq_kv_rollback(const int32_t* base, const int32_t* n_accepted, int B, int limit, int32_t* len,

@@ -227,6 +227,59 @@ __global__ void __launch_bounds__(kGemvThreads, (GemvMinBlocks<WK, MR, R, SILU>:
       if (base + b * kGemvThreads < total) xs[base + b * kGemvThreads] = v[b];
   }
   __syncthreads();
+  if (a.gamma != nullptr) {
+    // RMSNorm of the staged rows (x / sqrt(mean(x^2) + eps) * gamma, fp16
+    // out) in the arithmetic order of the standalone RMSNorm kernel: thread t
+    // sums the squares of k = t, t + 256, ..., then warp sums, then the eight
+    // warp sums in order, so the normalised rows equal its output bit for bit
+    __shared__ float nred[kGemvWarps * kGemvMaxRows];
+    __shared__ float rinv[kGemvMaxRows];
+    const __half* xh = reinterpret_cast<const __half*>(xs);
+    constexpr int WPP = 8 * SUB;  // weights (and x values) per 16-byte piece
+    for (int m = 0; m < MR; ++m) {
+      float ss = 0.0f;
+      if (m < a.M)
+        for (int k = threadIdx.x; k < (int)a.K; k += kGemvThreads) {
+          const int p = k / WPP, i = (k % WPP) >> 3;
+          const int slot = m * chunks_per_m + ((p >> 5) * SUB + i) * 32 + (p & 31);
+          const float v = __half2float(xh[slot * 8 + (k & 7)]);
+          ss = fmaf(v, v, ss);
+        }
+      ss = warp_sum(ss);
+      if ((threadIdx.x & 31) == 0) nred[(threadIdx.x >> 5) * kGemvMaxRows + m] = ss;
+    }
+    __syncthreads();
+    if (threadIdx.x < MR) {
+      float t = 0.0f;
+      for (int w = 0; w < kGemvWarps; ++w) t += nred[w * kGemvMaxRows + threadIdx.x];
+      rinv[threadIdx.x] = 1.0f / sqrtf(t / (float)a.K + a.eps);
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < total; idx += kGemvThreads) {
+      const int m = idx / chunks_per_m;
+      const int s = idx - m * chunks_per_m;
+      const int t = s >> 5, l = s & 31;
+      const int j = t / SUB, i = t - j * SUB;
+      const int p = j * 32 + l;
+      if (m >= a.M || p >= a.pieces) continue;
+      const uint4 g = *reinterpret_cast<const uint4*>(a.gamma + ((int64_t)p * SUB + i) * 8);
+      uint4 q = xs[idx];
+      const float r = rinv[m];
+      uint32_t* qw = reinterpret_cast<uint32_t*>(&q);
+      const uint32_t* gw = reinterpret_cast<const uint32_t*>(&g);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float lo = __fmul_rn(__fmul_rn(__half2float(__ushort_as_half(lo16(qw[e]))), r),
+                                   __half2float(__ushort_as_half(lo16(gw[e]))));
+        const float hi = __fmul_rn(__fmul_rn(__half2float(__ushort_as_half(hi16(qw[e]))), r),
+                                   __half2float(__ushort_as_half(hi16(gw[e]))));
+        qw[e] = (uint32_t)__half_as_ushort(__float2half_rn(lo)) |
+                ((uint32_t)__half_as_ushort(__float2half_rn(hi)) << 16);
+      }
+      xs[idx] = q;
+    }
+    __syncthreads();
+  }
   // INT4: per (row m, piece p) the offset 1032 X_even + 72 X_odd that the
   // magic-valued products carry (X = the piece's 32 activations summed over
   // even / odd k), behind x in shared memory

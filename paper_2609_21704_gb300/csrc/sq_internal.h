@@ -64,6 +64,8 @@ struct GemvArgs {
   int64_t row_bytes;       // bytes of one weight row
   int pieces;              // 16-byte pieces per weight row
   int ppad;                // pieces rounded up to a multiple of 32
+  const __half* gamma;     // [K] RMSNorm gains: x is normalised while staged; null = x as is
+  float eps;
 };
 constexpr int kGemvMaxRows = 16;
 size_t gemv_smem_bytes(int wkind, int mr, int64_t K);

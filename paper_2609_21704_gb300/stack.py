@@ -243,7 +243,8 @@ class DecoderState:
 
 
 def decoder_pass(stack: LinearStack, variant: str, st: DecoderState, stream=None,
-                 logits=None, pos0=None, last_only: bool = False, with_logits: bool = True) -> None:
+                 logits=None, pos0=None, last_only: bool = False, with_logits: bool = True,
+                 fused: bool = True) -> None:
     """One decoder step (draft or verify) with the variant's weights: per
     layer x += o(attn(rope(qkv(norm(x))))), x += down(silu-gate(norm(x)));
     then logits = lm_head(norm(x)) (into `logits` when given).  The new
@@ -251,24 +252,38 @@ def decoder_pass(stack: LinearStack, variant: str, st: DecoderState, stream=None
     reads them.  pos0 (int32 [B], device) overrides st.pos0; last_only
     runs the lm_head on each sequence's last token only (logits [B, V]);
     with_logits=False stops after the layers (a prefill that only fills
-    the cache)."""
-    from . import SQ_EPI_RESIDUAL, sq_attention, sq_embed, sq_kv_append, sq_rmsnorm
+    the cache).  fused: each RMSNorm runs inside the projection that reads
+    it (sq_linear_norm) and the cache append inside the attention
+    (sq_attention_append), five launches per layer instead of nine; the
+    results are bit-identical either way."""
+    from . import (SQ_EPI_RESIDUAL, sq_attention, sq_attention_append, sq_embed, sq_kv_append,
+                   sq_linear_norm, sq_rmsnorm)
     sh = stack.shape
     wk = WKIND[variant]
     B, T = st.B, st.T
     pos = st.pos0 if pos0 is None else pos0
+
+    def normed(x, gamma, h, w, s, epi, y):
+        if fused:
+            sq_linear_norm(wk, x, gamma, RMS_EPS, h, w, s, None, None, epi, y, stream)
+        else:
+            sq_rmsnorm(x, gamma, RMS_EPS, h, stream)
+            sq_linear_ex(wk, h, w, s, None, None, epi, y, stream)
+
     for li, (qkv, o, gu, down) in enumerate(stack.layers):
-        sq_rmsnorm(st.x, st.gamma[2 * li], RMS_EPS, st.h, stream)
         w, s = qkv.weight(variant)
-        sq_linear_ex(wk, st.h, w, s, None, None, SQ_EPI_NONE, st.qkv, stream)
-        sq_kv_append(st.qkv, B, T, sh.q_heads, sh.kv_heads, pos, ROPE_THETA, st.k[li], st.v[li], stream)
-        sq_attention(st.qkv, B, T, sh.q_heads, sh.kv_heads, pos, ROPE_THETA, st.k[li], st.v[li],
-                     st.attn, st.ws, stream)
+        normed(st.x, st.gamma[2 * li], st.h, w, s, SQ_EPI_NONE, st.qkv)
+        if fused:
+            sq_attention_append(st.qkv, B, T, sh.q_heads, sh.kv_heads, pos, ROPE_THETA, st.k[li], st.v[li],
+                                st.attn, st.ws, stream)
+        else:
+            sq_kv_append(st.qkv, B, T, sh.q_heads, sh.kv_heads, pos, ROPE_THETA, st.k[li], st.v[li], stream)
+            sq_attention(st.qkv, B, T, sh.q_heads, sh.kv_heads, pos, ROPE_THETA, st.k[li], st.v[li],
+                         st.attn, st.ws, stream)
         w, s = o.weight(variant)
         sq_linear_ex(wk, st.attn, w, s, None, st.x, SQ_EPI_RESIDUAL, st.x, stream)
-        sq_rmsnorm(st.x, st.gamma[2 * li + 1], RMS_EPS, st.h, stream)
         w, s = gu.weight(variant)
-        sq_linear_ex(wk, st.h, w, s, None, None, SQ_EPI_SILU_GATE, st.g, stream)
+        normed(st.x, st.gamma[2 * li + 1], st.h, w, s, SQ_EPI_SILU_GATE, st.g)
         w, s = down.weight(variant)
         sq_linear_ex(wk, st.g, w, s, None, st.x, SQ_EPI_RESIDUAL, st.x, stream)
     if stack.lm_head is None or not with_logits:
@@ -277,6 +292,5 @@ def decoder_pass(stack: LinearStack, variant: str, st: DecoderState, stream=None
     if last_only and T > 1:
         sq_embed(st.last_rows, st.x, st.x_last, stream)   # row gather
         x, h = st.x_last, st.h[:B]
-    sq_rmsnorm(x, st.gamma[-1], RMS_EPS, h, stream)
     w, s = stack.lm_head.weight(variant)
-    sq_linear_ex(wk, h, w, s, None, None, SQ_EPI_NONE, st.logits if logits is None else logits, stream)
+    normed(x, st.gamma[-1], h, w, s, SQ_EPI_NONE, st.logits if logits is None else logits)

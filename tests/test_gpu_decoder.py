@@ -114,3 +114,45 @@ def test_embed_gathers_rows_exactly():
     assert sq.sq_check() & sq.SQ_DEV_BAD_TOKEN_ID
     assert np.array_equal(out2[0].cpu().numpy().view(np.uint16), table[5].view(np.uint16))
     assert bool((out2[1] == 0).all())
+
+
+@pytest.mark.parametrize("B,T,Hq,Hkv,pos0,max_ctx", [
+    (2, 5, 12, 2, [37, 300], 512),      # new tokens straddle a 32-key chunk boundary in b = 0
+    (1, 1, 12, 2, [1023], 1024),        # last position of the cache
+    (3, 9, 28, 4, [64, 127, 700], 1024),
+    (1, 17, 12, 2, [0], 64),            # empty prefix, two chunks of new tokens
+    (4, 2, 40, 8, [30, 31, 32, 33], 96),
+])
+def test_fused_append_equals_append_then_attention(B, T, Hq, Hkv, pos0, max_ctx):
+    rng = np.random.default_rng(B * 1000 + T)
+    width = (Hq + 2 * Hkv) * D
+    qkv = _t(rng.normal(0, 1, (B * T, width)).astype(np.float16))
+    kc, vc = _fill_prefix(rng, B, Hkv, max_ctx, pos0)
+    p0 = _t(np.array(pos0, np.int32))
+    ws = torch.empty(sq.sq_attention_workspace_bytes(B, T, Hq, Hkv, max_ctx), dtype=torch.uint8,
+                     device=dev())
+    k1, v1 = _t(kc), _t(vc)
+    out1 = torch.empty(B * T, Hq * D, dtype=torch.float16, device=dev())
+    sq.sq_kv_append(qkv, B, T, Hq, Hkv, p0, THETA, k1, v1)
+    sq.sq_attention(qkv, B, T, Hq, Hkv, p0, THETA, k1, v1, out1, ws)
+    k2, v2 = _t(kc), _t(vc)
+    out2 = torch.empty(B * T, Hq * D, dtype=torch.float16, device=dev())
+    sq.sq_attention_append(qkv, B, T, Hq, Hkv, p0, THETA, k2, v2, out2, ws)
+    assert sq.sq_check() == 0
+    assert torch.equal(k1.view(torch.int16), k2.view(torch.int16))
+    assert torch.equal(v1.view(torch.int16), v2.view(torch.int16))
+    assert torch.equal(out1.view(torch.int16), out2.view(torch.int16))
+
+
+def test_fused_append_outside_the_cache_sets_status_and_writes_nothing():
+    B, T, Hq, Hkv, max_ctx = 1, 3, 12, 2, 64
+    qkv = torch.ones(B * T, (Hq + 2 * Hkv) * D, dtype=torch.float16, device=dev())
+    kc = torch.zeros(B, Hkv, max_ctx, D, dtype=torch.float16, device=dev())
+    vc = torch.zeros_like(kc)
+    out = torch.empty(B * T, Hq * D, dtype=torch.float16, device=dev())
+    ws = torch.empty(sq.sq_attention_workspace_bytes(B, T, Hq, Hkv, max_ctx), dtype=torch.uint8,
+                     device=dev())
+    sq.sq_attention_append(qkv, B, T, Hq, Hkv, _t(np.array([62], np.int32)), THETA, kc, vc, out, ws)
+    assert sq.sq_check() & sq.SQ_DEV_BAD_POSITION
+    assert not bool(kc.any()) and not bool(vc.any())
+    assert not bool(out.any())

@@ -62,3 +62,32 @@ def test_one_layer_matches_oracle_composition(variant, T):
     gact = _r16(oracle.silu_gate(full[:, :I], full[:, I:]))
     x2 = x1 + oracle.linear(gact, _w64(down_p, variant))
     assert_close(st.x.float().cpu().numpy().astype(np.float64), x2, f"{variant} layer output")
+
+
+@pytest.mark.parametrize("variant,T,last_only", [("int4", 1, False), ("int4", 2, True), ("fp16", 5, False),
+                                                 ("fp8", 3, True)])
+def test_fused_pass_equals_unfused(variant, T, last_only):
+    # sq_linear_norm and sq_attention_append are bit-identical to the calls
+    # they replace, so two layers plus the lm_head must agree exactly
+    sh = QWEN25_1P5B
+    S = stk.LinearStack(sh, dev(), seed=3, variants=("int4", "fp8"), layers=2)
+    B, max_ctx = 2, 256
+    rng = np.random.default_rng(12)
+    states = [stk.DecoderState(S, B, T, max_ctx, 0, seed=4) for _ in range(2)]
+    pre = [rng.normal(0, 1, (B, sh.kv_heads, 100, 128)).astype(np.float16) for _ in range(4)]
+    for st in states:
+        st.pos0.copy_(torch.tensor([100, 37], dtype=torch.int32))
+        for li in range(2):
+            st.k[li][:, :, :100] = torch.from_numpy(pre[2 * li]).to(dev())
+            st.v[li][:, :, :100] = torch.from_numpy(pre[2 * li + 1]).to(dev())
+    rows = B if last_only else B * T
+    out = [torch.empty(rows, sh.vocab, dtype=torch.float16, device=dev()) for _ in range(2)]
+    stk.decoder_pass(S, variant, states[0], logits=out[0], last_only=last_only, fused=True)
+    stk.decoder_pass(S, variant, states[1], logits=out[1], last_only=last_only, fused=False)
+    torch.cuda.synchronize()
+    a, b = states
+    assert torch.equal(out[0].view(torch.int16), out[1].view(torch.int16))
+    assert torch.equal(a.x.view(torch.int16), b.x.view(torch.int16))
+    for li in range(2):
+        assert torch.equal(a.k[li].view(torch.int16), b.k[li].view(torch.int16))
+        assert torch.equal(a.v[li].view(torch.int16), b.v[li].view(torch.int16))
