@@ -428,6 +428,7 @@ cudaError_t launch_gemv_inst(const GemvArgs& a, int64_t blocks_needed, size_t sm
   auto k = gemv_kernel<WK, MR, R, SILU, LPR>;
   struct Cached {
     int smem_set = 0;
+    int static_smem = -1;  // the kernel's static shared memory (bytes)
     size_t occ_smem[8] = {0};
     int occ[8] = {0};
   };
@@ -437,7 +438,14 @@ cudaError_t launch_gemv_inst(const GemvArgs& a, int64_t blocks_needed, size_t sm
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   Cached& c = cache[dev];
-  if (smem > 48 * 1024 && (int)smem > c.smem_set) {
+  if (c.static_smem < 0) {
+    cudaFuncAttributes fa;
+    e = cudaFuncGetAttributes(&fa, k);
+    if (e != cudaSuccess) return e;
+    c.static_smem = (int)fa.sharedSizeBytes;
+  }
+  // static + dynamic above the 48 KB default needs the opt-in attribute
+  if (smem + (size_t)c.static_smem > 48 * 1024 && (int)smem > c.smem_set) {
     e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     c.smem_set = (int)smem;

@@ -254,7 +254,7 @@ def decoder_pass(stack: LinearStack, variant: str, st: DecoderState, stream=None
     with_logits=False stops after the layers (a prefill that only fills
     the cache).  fused: each RMSNorm runs inside the projection that reads
     it (sq_linear_norm) and the cache append inside the attention
-    (sq_attention_append), five launches per layer instead of nine; the
+    (sq_attention_append), six launches per layer instead of nine; the
     results are bit-identical either way."""
     from . import (SQ_EPI_RESIDUAL, sq_attention, sq_attention_append, sq_embed, sq_kv_append,
                    sq_linear_norm, sq_rmsnorm)
