@@ -473,7 +473,9 @@ def main():
 
         g_ddu = capture(lambda: stk.decoder_pass(stack, args.draft, dd, stream, fused=False))
         t_ddu = timed(g_ddu, reps) / reps
-        del g_ddu
+        g_dvu = capture(lambda: stk.decoder_pass(stack, "fp16", dv, stream, fused=False))
+        t_dvu = timed(g_dvu, reps) / reps
+        del g_ddu, g_dvu
         g_dd = capture(lambda: stk.decoder_pass(stack, args.draft, dd, stream))
         g_dv = capture(lambda: stk.decoder_pass(stack, "fp16", dv, stream))
         g_dc = capture(dec_cycle)
@@ -649,6 +651,7 @@ def main():
             "decoder_context": ctx,
             "decoder_draft_pass_ms": 1e3 * t_dd,
             "decoder_draft_pass_unfused_ms": 1e3 * t_ddu,
+            "decoder_verify_pass_unfused_ms": 1e3 * t_dvu,
             "decoder_verify_pass_ms": 1e3 * t_dv,
             "decoder_cycle_ms": 1e3 * t_dc,
             "decoder_tokens_per_s": B * world * mean_tokens / t_dc,

@@ -49,11 +49,27 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const __half* __restrict__
   __shared__ float red[8];
   const int64_t m = blockIdx.x;
   const __half* xr = x + m * H;
+  // sum of squares over 8-value chunks: thread t takes chunks c = t, t + 256,
+  // ..., the values of a chunk in order (the order the projections that
+  // normalise their own staged rows use, so both give the same bits)
   float ss = 0.0f;
-  for (int64_t h = threadIdx.x; h < H; h += blockDim.x) {
-    const float v = __half2float(xr[h]);
-    ss = fmaf(v, v, ss);
+  const int64_t nch = H / 8;
+  const bool vec = (reinterpret_cast<uintptr_t>(xr) & 15) == 0;
+  for (int64_t c = threadIdx.x; c < nch; c += blockDim.x) {
+    if (vec) {
+      ss = sumsq8(reinterpret_cast<const uint4*>(xr)[c], ss);
+    } else {
+      for (int e = 0; e < 8; ++e) {
+        const float v = __half2float(xr[8 * c + e]);
+        ss = fmaf(v, v, ss);
+      }
+    }
   }
+  if (threadIdx.x == nch % blockDim.x)  // the ragged tail chunk (H % 8 values)
+    for (int64_t h = 8 * nch; h < H; ++h) {
+      const float v = __half2float(xr[h]);
+      ss = fmaf(v, v, ss);
+    }
   ss = warp_sum(ss);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
   __syncthreads();

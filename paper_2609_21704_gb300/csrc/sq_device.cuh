@@ -52,6 +52,21 @@ __device__ __forceinline__ float fma_h(uint16_t a, uint16_t b, float c) {
 __device__ __forceinline__ uint16_t lo16(uint32_t v) { return (uint16_t)(v & 0xffffu); }
 __device__ __forceinline__ uint16_t hi16(uint32_t v) { return (uint16_t)(v >> 16); }
 
+// ss + x0^2 + x1^2 + ... + x7^2 (fp32 fused multiply-adds in element order)
+// for eight fp16 values packed low half first: the RMSNorm sum of squares
+// takes each 8-value chunk of a row in this order.
+__device__ __forceinline__ float sumsq8(const uint4 q, float ss) {
+  const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float lo = __half2float(__ushort_as_half(lo16(w[e])));
+    const float hi = __half2float(__ushort_as_half(hi16(w[e])));
+    ss = fmaf(lo, lo, ss);
+    ss = fmaf(hi, hi, ss);
+  }
+  return ss;
+}
+
 // Two E4M3 codes (low byte -> low half) to two fp16 values (exact: every
 // E4M3 value is an fp16 value).
 __device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint16_t codes) {

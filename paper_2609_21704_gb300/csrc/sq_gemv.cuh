@@ -197,6 +197,10 @@ __global__ void __launch_bounds__(kGemvThreads, (GemvMinBlocks<WK, MR, R, SILU>:
 #pragma unroll
   for (int d = 1; d <= kPrefetchTiles; ++d) prefetch_tile(gwarp + (int64_t)d * nwarps);
   if (gwarp < t_end) load_batch(gwarp, 0);
+  // the RMSNorm gains never depend on it either: bring this thread's first
+  // chunk into L1 (the weight loads do not allocate there)
+  if (a.gamma != nullptr && threadIdx.x < a.K / 8)
+    asm volatile("prefetch.global.L1 [%0];" ::"l"(a.gamma + 8 * threadIdx.x));
 
   griddep_wait();
   griddep_launch_dependents();
@@ -230,21 +234,20 @@ __global__ void __launch_bounds__(kGemvThreads, (GemvMinBlocks<WK, MR, R, SILU>:
   if (a.gamma != nullptr) {
     // RMSNorm of the staged rows (x / sqrt(mean(x^2) + eps) * gamma, fp16
     // out) in the arithmetic order of the standalone RMSNorm kernel: thread t
-    // sums the squares of k = t, t + 256, ..., then warp sums, then the eight
-    // warp sums in order, so the normalised rows equal its output bit for bit
+    // sums the 8-value chunks c = t, t + 256, ... (values in order), then warp
+    // sums, then the eight warp sums in order; so the normalised rows equal
+    // its output bit for bit.  A chunk is one staged 16-byte slot.
     __shared__ float nred[kGemvWarps * kGemvMaxRows];
     __shared__ float rinv[kGemvMaxRows];
-    const __half* xh = reinterpret_cast<const __half*>(xs);
-    constexpr int WPP = 8 * SUB;  // weights (and x values) per 16-byte piece
+    const int nch = (int)(a.K / 8);
+    auto chunk_slot = [&](int c) {
+      const int p = c / SUB, i = c - (c / SUB) * SUB;
+      return ((p >> 5) * SUB + i) * 32 + (p & 31);
+    };
     for (int m = 0; m < MR; ++m) {
       float ss = 0.0f;
       if (m < a.M)
-        for (int k = threadIdx.x; k < (int)a.K; k += kGemvThreads) {
-          const int p = k / WPP, i = (k % WPP) >> 3;
-          const int slot = m * chunks_per_m + ((p >> 5) * SUB + i) * 32 + (p & 31);
-          const float v = __half2float(xh[slot * 8 + (k & 7)]);
-          ss = fmaf(v, v, ss);
-        }
+        for (int c = threadIdx.x; c < nch; c += kGemvThreads) ss = sumsq8(xs[m * chunks_per_m + chunk_slot(c)], ss);
       ss = warp_sum(ss);
       if ((threadIdx.x & 31) == 0) nred[(threadIdx.x >> 5) * kGemvMaxRows + m] = ss;
     }
@@ -255,28 +258,25 @@ __global__ void __launch_bounds__(kGemvThreads, (GemvMinBlocks<WK, MR, R, SILU>:
       rinv[threadIdx.x] = 1.0f / sqrtf(t / (float)a.K + a.eps);
     }
     __syncthreads();
-    for (int idx = threadIdx.x; idx < total; idx += kGemvThreads) {
-      const int m = idx / chunks_per_m;
-      const int s = idx - m * chunks_per_m;
-      const int t = s >> 5, l = s & 31;
-      const int j = t / SUB, i = t - j * SUB;
-      const int p = j * 32 + l;
-      if (m >= a.M || p >= a.pieces) continue;
-      const uint4 g = *reinterpret_cast<const uint4*>(a.gamma + ((int64_t)p * SUB + i) * 8);
-      uint4 q = xs[idx];
-      const float r = rinv[m];
-      uint32_t* qw = reinterpret_cast<uint32_t*>(&q);
-      const uint32_t* gw = reinterpret_cast<const uint32_t*>(&g);
+    for (int c = threadIdx.x; c < nch; c += kGemvThreads) {
+      const int slot = chunk_slot(c);
+      const uint4 g = *reinterpret_cast<const uint4*>(a.gamma + 8 * (int64_t)c);
+      const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
+      for (int m = 0; m < MR && m < a.M; ++m) {
+        uint4 q = xs[m * chunks_per_m + slot];
+        uint32_t* qw = reinterpret_cast<uint32_t*>(&q);
+        const float r = rinv[m];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float lo = __fmul_rn(__fmul_rn(__half2float(__ushort_as_half(lo16(qw[e]))), r),
-                                   __half2float(__ushort_as_half(lo16(gw[e]))));
-        const float hi = __fmul_rn(__fmul_rn(__half2float(__ushort_as_half(hi16(qw[e]))), r),
-                                   __half2float(__ushort_as_half(hi16(gw[e]))));
-        qw[e] = (uint32_t)__half_as_ushort(__float2half_rn(lo)) |
-                ((uint32_t)__half_as_ushort(__float2half_rn(hi)) << 16);
+        for (int e = 0; e < 4; ++e) {
+          const float lo = __fmul_rn(__fmul_rn(__half2float(__ushort_as_half(lo16(qw[e]))), r),
+                                     __half2float(__ushort_as_half(lo16(gw[e]))));
+          const float hi = __fmul_rn(__fmul_rn(__half2float(__ushort_as_half(hi16(qw[e]))), r),
+                                     __half2float(__ushort_as_half(hi16(gw[e]))));
+          qw[e] = (uint32_t)__half_as_ushort(__float2half_rn(lo)) |
+                  ((uint32_t)__half_as_ushort(__float2half_rn(hi)) << 16);
+        }
+        xs[m * chunks_per_m + slot] = q;
       }
-      xs[idx] = q;
     }
     __syncthreads();
   }
