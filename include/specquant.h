@@ -313,7 +313,7 @@ SQ_API sq_status sq_softmax(const void* z, int64_t R, int64_t V, float temperatu
  * projection's output for T new tokens of each of B sequences (row b*T + t:
  * q heads, then k heads, then v heads); D = 128; Hq a multiple of Hkv; token
  * t of sequence b is at position pos0[b] + t (pos0 int32 [B], device).
- * Caches k_cache, v_cache fp16 [B, Hkv, max_ctx, D].  RoPE rotates pairs
+ * Caches k_cache, v_cache fp16 [B, Hkv, max_ctx, D], 16-byte aligned.  RoPE rotates pairs
  * (d, d + D/2) by pos * theta^(-2d/D) (angle computed in fp64).
  *
  * sq_kv_append: rotates the new keys and writes keys and values into the

@@ -136,6 +136,9 @@ __global__ void __launch_bounds__(64) kv_append_kernel(const __half* __restrict_
 }
 
 // ---- attention ----------------------------------------------------------------
+__device__ __forceinline__ float h2f_lo(uint32_t w) { return __half2float(__ushort_as_half((uint16_t)(w & 0xffffu))); }
+__device__ __forceinline__ float h2f_hi(uint32_t w) { return __half2float(__ushort_as_half((uint16_t)(w >> 16))); }
+
 struct AttnArgs {
   const __half* qkv;
   const __half* kc;
@@ -184,41 +187,62 @@ __global__ void __launch_bounds__(kAttnThreads) attention_partial_kernel(const A
   }
   const int nk = (int)(len - j0 < kAttnChunk ? len - j0 : kAttnChunk);
   const int64_t width = (int64_t)(a.Hq + 2 * a.Hkv) * kHeadDim;
-  for (int idx = tid; idx < T * (kHeadDim / 2); idx += kAttnThreads) {
-    const int t = idx / (kHeadDim / 2), d = idx - t * (kHeadDim / 2);
-    cst[idx] = rope_cs(p0 + t, a.rf.f[d]);
-  }
   const int64_t cbase = (((int64_t)b * a.Hkv + kvh) * a.max_ctx + j0) * kHeadDim;
   // positions p0 .. p0+T-1 are the new tokens: with append, this chunk's
   // share of them is rotated from qkv, written to the caches and used
   // directly (every position belongs to one chunk, so each is written once)
   const int j_new = a.append ? (int)((int64_t)p0 - j0) : kAttnChunk;  // first new key of the chunk
-  if (j_new < nk) __syncthreads();  // cst is read below
-  for (int idx = tid; idx < kAttnChunk * kHeadDim; idx += kAttnThreads) {
-    const int j = idx / kHeadDim, d = idx - j * kHeadDim;
-    float kf = 0.0f, vf = 0.0f;
-    if (j < nk) {
-      if (j >= j_new) {
-        const int t = (int)(j0 + j - p0);
-        const __half* row = a.qkv + ((int64_t)b * T + t) * width;
-        const __half* kr = row + (int64_t)(a.Hq + kvh) * kHeadDim;
-        const __half vh = row[(int64_t)(a.Hq + a.Hkv + kvh) * kHeadDim + d];
-        const int pd = d & (kHeadDim / 2 - 1);
-        __half y1, y2;
-        rope_rotate_f16(__half2float(kr[pd]), __half2float(kr[pd + kHeadDim / 2]),
-                        cst[t * (kHeadDim / 2) + pd], y1, y2);
-        const __half kh = d < kHeadDim / 2 ? y1 : y2;
-        a.kcw[cbase + idx] = kh;
-        a.vcw[cbase + idx] = vh;
-        kf = __half2float(kh);
-        vf = __half2float(vh);
-      } else {
-        kf = __half2float(a.kc[cbase + idx]);
-        vf = __half2float(a.vc[cbase + idx]);
-      }
+  const int n_old = j_new < nk ? (j_new > 0 ? j_new : 0) : nk;         // keys read from the caches
+  // cached keys and values: 16-byte pieces (8 values), all of a thread's
+  // loads issued before the RoPE table is computed
+  constexpr int kPieces = kAttnChunk * kHeadDim / 8;
+  constexpr int kPerThread = kPieces / kAttnThreads;
+  static_assert(kPieces % kAttnThreads == 0, "whole pieces per thread");
+  uint4 kraw[kPerThread], vraw[kPerThread];
+#pragma unroll
+  for (int r = 0; r < kPerThread; ++r) {
+    const int pc = tid + r * kAttnThreads;
+    const int j = pc / (kHeadDim / 8);
+    const bool in = j < n_old;
+    kraw[r] = in ? *reinterpret_cast<const uint4*>(a.kc + cbase + (int64_t)pc * 8) : make_uint4(0u, 0u, 0u, 0u);
+    vraw[r] = in ? *reinterpret_cast<const uint4*>(a.vc + cbase + (int64_t)pc * 8) : make_uint4(0u, 0u, 0u, 0u);
+  }
+  for (int idx = tid; idx < T * (kHeadDim / 2); idx += kAttnThreads) {
+    const int t = idx / (kHeadDim / 2), d = idx - t * (kHeadDim / 2);
+    cst[idx] = rope_cs(p0 + t, a.rf.f[d]);
+  }
+#pragma unroll
+  for (int r = 0; r < kPerThread; ++r) {
+    const int pc = tid + r * kAttnThreads;
+    const int j = pc / (kHeadDim / 8), d8 = pc - j * (kHeadDim / 8);
+    if (j >= n_old && j < nk) continue;  // a new key: written below
+    const uint32_t kw[4] = {kraw[r].x, kraw[r].y, kraw[r].z, kraw[r].w};
+    const uint32_t vw[4] = {vraw[r].x, vraw[r].y, vraw[r].z, vraw[r].w};
+    float4* kd = reinterpret_cast<float4*>(ks + j * kRowPad + d8 * 8);
+    float4* vd = reinterpret_cast<float4*>(vs + j * kRowPad + d8 * 8);
+    kd[0] = make_float4(h2f_lo(kw[0]), h2f_hi(kw[0]), h2f_lo(kw[1]), h2f_hi(kw[1]));
+    kd[1] = make_float4(h2f_lo(kw[2]), h2f_hi(kw[2]), h2f_lo(kw[3]), h2f_hi(kw[3]));
+    vd[0] = make_float4(h2f_lo(vw[0]), h2f_hi(vw[0]), h2f_lo(vw[1]), h2f_hi(vw[1]));
+    vd[1] = make_float4(h2f_lo(vw[2]), h2f_hi(vw[2]), h2f_lo(vw[3]), h2f_hi(vw[3]));
+  }
+  if (n_old < nk) {  // new keys of this chunk (append): rotate from qkv
+    __syncthreads();  // cst is read below
+    for (int idx = n_old * kHeadDim + tid; idx < nk * kHeadDim; idx += kAttnThreads) {
+      const int j = idx / kHeadDim, d = idx - j * kHeadDim;
+      const int t = (int)(j0 + j - p0);
+      const __half* row = a.qkv + ((int64_t)b * T + t) * width;
+      const __half* kr = row + (int64_t)(a.Hq + kvh) * kHeadDim;
+      const __half vh = row[(int64_t)(a.Hq + a.Hkv + kvh) * kHeadDim + d];
+      const int pd = d & (kHeadDim / 2 - 1);
+      __half y1, y2;
+      rope_rotate_f16(__half2float(kr[pd]), __half2float(kr[pd + kHeadDim / 2]), cst[t * (kHeadDim / 2) + pd],
+                      y1, y2);
+      const __half kh = d < kHeadDim / 2 ? y1 : y2;
+      a.kcw[cbase + idx] = kh;
+      a.vcw[cbase + idx] = vh;
+      ks[j * kRowPad + d] = __half2float(kh);
+      vs[j * kRowPad + d] = __half2float(vh);
     }
-    ks[j * kRowPad + d] = kf;
-    vs[j * kRowPad + d] = vf;
   }
   __syncthreads();
   for (int idx = tid; idx < Q * (kHeadDim / 2); idx += kAttnThreads) {

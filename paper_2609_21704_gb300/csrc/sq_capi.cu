@@ -467,8 +467,8 @@ static sq_status check_attn(const char* who, const void* qkv, int B, int T, int 
   if (!(theta > 1.0f) || !std::isfinite(theta)) return fail(SQ_ERR_INVALID_ARG, "%s: theta must be > 1", who);
   if (B > 0 && T > 0 && (!qkv || !pos0 || !kc || !vc))
     return fail(SQ_ERR_INVALID_ARG, "%s: NULL pointer", who);
-  if (!aligned(qkv, 2) || !aligned(pos0, 4) || !aligned(kc, 2) || !aligned(vc, 2))
-    return fail(SQ_ERR_ALIGN, "%s: misaligned pointer", who);
+  if (!aligned(qkv, 2) || !aligned(pos0, 4) || !aligned(kc, 16) || !aligned(vc, 16))
+    return fail(SQ_ERR_ALIGN, "%s: misaligned pointer (caches need 16 bytes)", who);
   return SQ_OK;
 }
 

@@ -244,7 +244,7 @@ class DecoderState:
 
 def decoder_pass(stack: LinearStack, variant: str, st: DecoderState, stream=None,
                  logits=None, pos0=None, last_only: bool = False, with_logits: bool = True,
-                 fused: bool = True) -> None:
+                 fused: bool = True, fuse_norm: bool | None = None, fuse_append: bool | None = None) -> None:
     """One decoder step (draft or verify) with the variant's weights: per
     layer x += o(attn(rope(qkv(norm(x))))), x += down(silu-gate(norm(x)));
     then logits = lm_head(norm(x)) (into `logits` when given).  The new
@@ -253,18 +253,24 @@ def decoder_pass(stack: LinearStack, variant: str, st: DecoderState, stream=None
     runs the lm_head on each sequence's last token only (logits [B, V]);
     with_logits=False stops after the layers (a prefill that only fills
     the cache).  fused: each RMSNorm runs inside the projection that reads
-    it (sq_linear_norm) and the cache append inside the attention
-    (sq_attention_append), six launches per layer instead of nine; the
-    results are bit-identical either way."""
+    it (sq_linear_norm) and, for one new token per sequence, the cache
+    append inside the attention (sq_attention_append): six launches per
+    layer instead of nine; the results are bit-identical either way
+    (fuse_norm / fuse_append override the two choices)."""
     from . import (SQ_EPI_RESIDUAL, sq_attention, sq_attention_append, sq_embed, sq_kv_append,
                    sq_linear_norm, sq_rmsnorm)
     sh = stack.shape
     wk = WKIND[variant]
     B, T = st.B, st.T
     pos = st.pos0 if pos0 is None else pos0
+    fuse_norm = fused if fuse_norm is None else fuse_norm
+    # the fused append measured faster in passes of one new token per
+    # sequence but slower from two on (the kernels launched after it lose
+    # overlap; 10 us per layer at five tokens), so it is the default at T = 1
+    fuse_append = (fused and T == 1) if fuse_append is None else fuse_append
 
     def normed(x, gamma, h, w, s, epi, y):
-        if fused:
+        if fuse_norm:
             sq_linear_norm(wk, x, gamma, RMS_EPS, h, w, s, None, None, epi, y, stream)
         else:
             sq_rmsnorm(x, gamma, RMS_EPS, h, stream)
@@ -273,7 +279,7 @@ def decoder_pass(stack: LinearStack, variant: str, st: DecoderState, stream=None
     for li, (qkv, o, gu, down) in enumerate(stack.layers):
         w, s = qkv.weight(variant)
         normed(st.x, st.gamma[2 * li], st.h, w, s, SQ_EPI_NONE, st.qkv)
-        if fused:
+        if fuse_append:
             sq_attention_append(st.qkv, B, T, sh.q_heads, sh.kv_heads, pos, ROPE_THETA, st.k[li], st.v[li],
                                 st.attn, st.ws, stream)
         else:

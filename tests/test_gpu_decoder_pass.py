@@ -82,7 +82,8 @@ def test_fused_pass_equals_unfused(variant, T, last_only):
             st.v[li][:, :, :100] = torch.from_numpy(pre[2 * li + 1]).to(dev())
     rows = B if last_only else B * T
     out = [torch.empty(rows, sh.vocab, dtype=torch.float16, device=dev()) for _ in range(2)]
-    stk.decoder_pass(S, variant, states[0], logits=out[0], last_only=last_only, fused=True)
+    stk.decoder_pass(S, variant, states[0], logits=out[0], last_only=last_only, fuse_norm=True,
+                     fuse_append=True)
     stk.decoder_pass(S, variant, states[1], logits=out[1], last_only=last_only, fused=False)
     torch.cuda.synchronize()
     a, b = states
