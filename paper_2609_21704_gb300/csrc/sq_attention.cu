@@ -245,14 +245,38 @@ __global__ void __launch_bounds__(kAttnThreads) attention_partial_kernel(const A
     }
   }
   __syncthreads();
-  for (int idx = tid; idx < Q * (kHeadDim / 2); idx += kAttnThreads) {
-    const int q = idx / (kHeadDim / 2), d = idx - q * (kHeadDim / 2);
+  // queries: each thread rotates 8 pairs (d, d + D/2) read as two 16-byte
+  // pieces (q rows are 16-byte aligned when qkv is: D = 128 halves)
+  const bool qvec = (reinterpret_cast<uintptr_t>(a.qkv) & 15) == 0;
+  for (int idx = tid; idx < Q * (kHeadDim / 16); idx += kAttnThreads) {
+    const int q = idx / (kHeadDim / 16), d0 = (idx - q * (kHeadDim / 16)) * 8;
     const int g = q / T, t = q - g * T;
     const __half* qr = a.qkv + ((int64_t)b * T + t) * width + (int64_t)(kvh * a.G + g) * kHeadDim;
-    const float2 cs = cst[t * (kHeadDim / 2) + d];
-    const float x1 = __half2float(qr[d]), x2 = __half2float(qr[d + kHeadDim / 2]);
-    qs[q * kRowPad + d] = (x1 * cs.x - x2 * cs.y) * a.scale;
-    qs[q * kRowPad + d + kHeadDim / 2] = (x2 * cs.x + x1 * cs.y) * a.scale;
+    float x1[8], x2[8];
+    if (qvec) {
+      const uint4 u1 = *reinterpret_cast<const uint4*>(qr + d0);
+      const uint4 u2 = *reinterpret_cast<const uint4*>(qr + d0 + kHeadDim / 2);
+      const uint32_t w1[4] = {u1.x, u1.y, u1.z, u1.w}, w2[4] = {u2.x, u2.y, u2.z, u2.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        x1[2 * e] = h2f_lo(w1[e]);
+        x1[2 * e + 1] = h2f_hi(w1[e]);
+        x2[2 * e] = h2f_lo(w2[e]);
+        x2[2 * e + 1] = h2f_hi(w2[e]);
+      }
+    } else {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        x1[e] = __half2float(qr[d0 + e]);
+        x2[e] = __half2float(qr[d0 + e + kHeadDim / 2]);
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const float2 cs = cst[t * (kHeadDim / 2) + d0 + e];
+      qs[q * kRowPad + d0 + e] = (x1[e] * cs.x - x2[e] * cs.y) * a.scale;
+      qs[q * kRowPad + d0 + e + kHeadDim / 2] = (x2[e] * cs.x + x1[e] * cs.y) * a.scale;
+    }
   }
   __syncthreads();
   // scores: each thread a 2-query x 4-key tile, 16-byte shared loads along D
@@ -345,12 +369,26 @@ __global__ void __launch_bounds__(kHeadDim) attention_combine_kernel(const AttnA
   for (int w = 0; w < kHeadDim / 32; ++w) M = fmaxf(M, red[w]);
   float L = 0.0f, O = 0.0f;
   if (M != -INFINITY)
-    for (int s = 0; s < a.nsplit; ++s) {
-      const float ms = cm[s];
-      if (ms == -INFINITY) continue;
-      const float w = expf(ms - M);
-      L = fmaf(w, cm[a.nsplit + s], L);
-      O = fmaf(w, base[((int64_t)s * a.Q + q) * kPartStride + kPartO + d], O);
+    for (int s0 = 0; s0 < a.nsplit; s0 += 8) {
+      // the chunks' weighted values, eight loads in flight; then the same
+      // sums, chunk by chunk in order
+      float ov[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int s = s0 + u;
+        ov[u] = (s < a.nsplit && cm[s] != -INFINITY) ? base[((int64_t)s * a.Q + q) * kPartStride + kPartO + d]
+                                                      : 0.0f;
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int s = s0 + u;
+        if (s >= a.nsplit) break;
+        const float ms = cm[s];
+        if (ms == -INFINITY) continue;
+        const float w = expf(ms - M);
+        L = fmaf(w, cm[a.nsplit + s], L);
+        O = fmaf(w, ov[u], O);
+      }
     }
   const int g = q / a.T, t = q - g * a.T;
   const int64_t row = (int64_t)b * a.T + t;

@@ -56,7 +56,10 @@ struct TcConv {
   static constexpr int threads = 64 + 32 * warps;
 };
 constexpr int kTcStageA = kTcBM * kTcBK * 2;  // 16 KB
-constexpr int kTcMaxSplit = 8;  // CTAs per cluster along K (portable cluster size)
+// CTAs per cluster along K: up to 16 (non-portable cluster size, allowed at
+// launch); the INT4 search keeps to the portable 8 it was measured at.
+constexpr int kTcMaxSplit = 16;
+constexpr int kTcMaxSplitInt4 = 8;
 
 // ---------------------------------------------------------------- PTX
 
@@ -589,16 +592,19 @@ static int tc_pick_split(int64_t tiles, int ksteps, size_t smem, int max_split, 
     const int sms = device_sm_count();
     int S = 1;
     if (two_per_sm) {
-      // two CTAs per SM: the largest S that still fits one wave
+      // two CTAs per SM: the largest S (up to 16, a cluster on 8 SMs) that
+      // still fits one wave (1.5B down projection, M = 5: 10.4 -> 8.7 us
+      // from S = 8 to 16)
       while (S < max_split && tiles * (S + 1) <= 2 * sms && ksteps >= 4 * (S + 1)) ++S;
       return S;
     }
-    while (2 * S <= max_split && tiles * S * 2 <= sms && ksteps >= 4 * S * 2) S <<= 1;
+    // one CTA per SM: clusters of at most the portable 8 SMs
+    while (2 * S <= max_split && 2 * S <= 8 && tiles * S * 2 <= sms && ksteps >= 4 * S * 2) S <<= 1;
     return S;
   }
   int best_s = 1;
   int64_t best = INT64_MAX;
-  for (int S = 1; S <= max_split && ksteps >= 2 * S; ++S) {
+  for (int S = 1; S <= max_split && S <= kTcMaxSplitInt4 && ksteps >= 2 * S; ++S) {
     const int nc = tc_max_clusters<WK, SILU>(S, smem);
     if (nc <= 0) continue;
     const int64_t waves = (tiles + nc - 1) / nc;
