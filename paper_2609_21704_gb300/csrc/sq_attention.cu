@@ -16,13 +16,10 @@
 // output rows [B*T, Hq D].  Token t of sequence b sits at position
 // pos0[b] + t.
 //
-// Attention runs over 32-key chunks of the cache.  Up to 64 queries per
-// group: one launch, a thread-block cluster per (sequence, key/value head)
-// whose CTAs share the chunks (online softmax) and merge through
-// distributed shared memory.  Larger groups: one CTA per (sequence,
-// key/value head, chunk), all G * T queries of the group reading the chunk
-// once from shared memory, then a combine kernel merging the chunks'
-// (max, sum, weighted value) partials.  Bound: the cache bytes
+// Attention is split over 64-key chunks of the cache (one CTA per
+// (sequence, key/value head, chunk)): all G * T queries of the group read
+// the chunk once from shared memory, then a combine kernel merges the
+// chunks' (max, sum, weighted value) partials.  Bound: the cache bytes
 // (2 * pos * Hkv * D * 2 per sequence) and, for long query groups, CUDA-core
 // arithmetic (G * T * 2 D flops per cached key).
 #include <math.h>
@@ -155,7 +152,6 @@ struct AttnArgs {
   int B, T, Hq, Hkv, G, Q;
   int64_t max_ctx;
   int nsplit;
-  int S;        // CTAs per cluster (one-launch kernel)
   float scale;  // 1 / sqrt(D)
   RopeFreq rf;
 };
@@ -400,282 +396,6 @@ __global__ void __launch_bounds__(kHeadDim) attention_combine_kernel(const AttnA
       __float2half_rn(L > 0.0f ? O / L : 0.0f);
 }
 
-// ---- attention in one launch: a cluster per (sequence, key/value head) ----------------
-// The S CTAs of a cluster take the 32-key chunks c = rank, rank + S, ... of
-// the sequence, each keeping an online softmax over its chunks (per query a
-// running maximum, sum and weighted value row, rescaled by exp(m_old -
-// m_new) when the maximum grows); the next chunk's keys and values are
-// loaded into registers while the current one is computed.  After a cluster
-// barrier CTA r merges the S states of queries q = r, r + S, ... read from
-// the other CTAs' shared memory (in rank order, so the result does not
-// depend on timing) and writes the output rows: no partials go through
-// global memory and there is no second launch.  Up to kClusterMaxQ queries
-// per group; every CTA reaches both cluster barriers.
-constexpr int kClusterMaxQ = 64;
-constexpr int kClusterMaxS = 8;  // portable cluster size
-
-__device__ __forceinline__ uint32_t attn_cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-__device__ __forceinline__ void attn_cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-__device__ __forceinline__ float attn_ld_dsmem(const float* local, uint32_t rank) {
-  const uint32_t la = (uint32_t)__cvta_generic_to_shared(local);
-  uint32_t remote;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(la), "r"(rank));
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
-  return v;
-}
-
-// Shared memory (fp32): cos/sin [T][D/2], q [Q][kRowPad] (rotated, scaled),
-// k, v [C][kRowPad], scores [Q][C], running weighted values [Q][kRowPad],
-// running maximum, sum and rescale factor [Q] each.
-size_t attention_cluster_smem_bytes(int T, int Q) {
-  return ((size_t)2 * T * (kHeadDim / 2) + (size_t)Q * kRowPad + (size_t)2 * kAttnChunk * kRowPad +
-          (size_t)Q * kAttnChunk + (size_t)Q * kRowPad + (size_t)3 * Q) *
-         sizeof(float);
-}
-
-__global__ void __launch_bounds__(kAttnThreads) attention_cluster_kernel(const AttnArgs a) {
-  griddep_wait();
-  griddep_launch_dependents();
-  extern __shared__ __align__(16) float sm[];
-  const int Q = a.Q, T = a.T, S = a.S;
-  float2* cst = reinterpret_cast<float2*>(sm);  // [T][D/2]
-  float* qs = sm + 2 * T * (kHeadDim / 2);       // [Q][kRowPad]
-  float* ks = qs + Q * kRowPad;                  // [C][kRowPad]
-  float* vs = ks + kAttnChunk * kRowPad;         // [C][kRowPad]
-  float* sc = vs + kAttnChunk * kRowPad;         // [Q][C]
-  float* os = sc + Q * kAttnChunk;               // [Q][kRowPad]
-  float* ms = os + Q * kRowPad;                  // [Q]
-  float* ls = ms + Q;                            // [Q]
-  float* al = ls + Q;                            // [Q]
-  const int bh = blockIdx.x;
-  const int b = bh / a.Hkv, kvh = bh - b * a.Hkv;
-  const int tid = threadIdx.x;
-  const uint32_t rank = attn_cluster_rank();
-  const int p0 = a.pos0[b];
-  const int64_t len = (int64_t)p0 + T;
-  const bool ok = p0 >= 0 && len <= a.max_ctx;
-  if (a.append && !ok && rank == 0 && tid == 0) atomicOr(&g_attn_status, SQ_DEV_BAD_POSITION);
-  const int nch = ok ? (int)((len + kAttnChunk - 1) / kAttnChunk) : 0;
-  const int64_t width = (int64_t)(a.Hq + 2 * a.Hkv) * kHeadDim;
-  const int64_t hbase = ((int64_t)b * a.Hkv + kvh) * a.max_ctx * kHeadDim;
-
-  for (int i = tid; i < Q * kRowPad; i += kAttnThreads) os[i] = 0.0f;
-  for (int q = tid; q < Q; q += kAttnThreads) {
-    ms[q] = -INFINITY;
-    ls[q] = 0.0f;
-  }
-  constexpr int kPieces = kAttnChunk * kHeadDim / 8;
-  constexpr int kPerThread = kPieces / kAttnThreads;
-  uint4 kraw[kPerThread], vraw[kPerThread];
-  // cached keys / values of chunk cc (positions before the new tokens when
-  // appending), 16-byte pieces
-  auto load_raw = [&](int cc) {
-    const int64_t j0 = (int64_t)cc * kAttnChunk;
-    const int nk = (int)(len - j0 < kAttnChunk ? len - j0 : kAttnChunk);
-    const int j_new = a.append ? (int)((int64_t)p0 - j0) : kAttnChunk;
-    const int n_old = j_new < nk ? (j_new > 0 ? j_new : 0) : nk;
-#pragma unroll
-    for (int r = 0; r < kPerThread; ++r) {
-      const int pc = tid + r * kAttnThreads;
-      const bool in = pc / (kHeadDim / 8) < n_old;
-      const int64_t off = hbase + j0 * kHeadDim + (int64_t)pc * 8;
-      kraw[r] = in ? *reinterpret_cast<const uint4*>(a.kc + off) : make_uint4(0u, 0u, 0u, 0u);
-      vraw[r] = in ? *reinterpret_cast<const uint4*>(a.vc + off) : make_uint4(0u, 0u, 0u, 0u);
-    }
-  };
-  int c = (int)rank;
-  if (c < nch) load_raw(c);
-  if (nch > 0) {
-    for (int idx = tid; idx < T * (kHeadDim / 2); idx += kAttnThreads) {
-      const int t = idx / (kHeadDim / 2), d = idx - t * (kHeadDim / 2);
-      cst[idx] = rope_cs(p0 + t, a.rf.f[d]);
-    }
-  }
-  __syncthreads();
-  if (c < nch) {
-    const bool qvec = (reinterpret_cast<uintptr_t>(a.qkv) & 15) == 0;
-    for (int idx = tid; idx < Q * (kHeadDim / 16); idx += kAttnThreads) {
-      const int q = idx / (kHeadDim / 16), d0 = (idx - q * (kHeadDim / 16)) * 8;
-      const int g = q / T, t = q - g * T;
-      const __half* qr = a.qkv + ((int64_t)b * T + t) * width + (int64_t)(kvh * a.G + g) * kHeadDim;
-      float x1[8], x2[8];
-      if (qvec) {
-        const uint4 u1 = *reinterpret_cast<const uint4*>(qr + d0);
-        const uint4 u2 = *reinterpret_cast<const uint4*>(qr + d0 + kHeadDim / 2);
-        const uint32_t w1[4] = {u1.x, u1.y, u1.z, u1.w}, w2[4] = {u2.x, u2.y, u2.z, u2.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          x1[2 * e] = h2f_lo(w1[e]);
-          x1[2 * e + 1] = h2f_hi(w1[e]);
-          x2[2 * e] = h2f_lo(w2[e]);
-          x2[2 * e + 1] = h2f_hi(w2[e]);
-        }
-      } else {
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          x1[e] = __half2float(qr[d0 + e]);
-          x2[e] = __half2float(qr[d0 + e + kHeadDim / 2]);
-        }
-      }
-#pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        const float2 cs = cst[t * (kHeadDim / 2) + d0 + e];
-        qs[q * kRowPad + d0 + e] = (x1[e] * cs.x - x2[e] * cs.y) * a.scale;
-        qs[q * kRowPad + d0 + e + kHeadDim / 2] = (x2[e] * cs.x + x1[e] * cs.y) * a.scale;
-      }
-    }
-  }
-  const int qpairs = (Q + 1) / 2;
-  while (c < nch) {
-    const int64_t j0 = (int64_t)c * kAttnChunk;
-    const int nk = (int)(len - j0 < kAttnChunk ? len - j0 : kAttnChunk);
-    const int j_new = a.append ? (int)((int64_t)p0 - j0) : kAttnChunk;
-    const int n_old = j_new < nk ? (j_new > 0 ? j_new : 0) : nk;
-#pragma unroll
-    for (int r = 0; r < kPerThread; ++r) {
-      const int pc = tid + r * kAttnThreads;
-      const int j = pc / (kHeadDim / 8), d8 = pc - j * (kHeadDim / 8);
-      if (j >= n_old && j < nk) continue;  // a new key: written below
-      const uint32_t kw[4] = {kraw[r].x, kraw[r].y, kraw[r].z, kraw[r].w};
-      const uint32_t vw[4] = {vraw[r].x, vraw[r].y, vraw[r].z, vraw[r].w};
-      float4* kd = reinterpret_cast<float4*>(ks + j * kRowPad + d8 * 8);
-      float4* vd = reinterpret_cast<float4*>(vs + j * kRowPad + d8 * 8);
-      kd[0] = make_float4(h2f_lo(kw[0]), h2f_hi(kw[0]), h2f_lo(kw[1]), h2f_hi(kw[1]));
-      kd[1] = make_float4(h2f_lo(kw[2]), h2f_hi(kw[2]), h2f_lo(kw[3]), h2f_hi(kw[3]));
-      vd[0] = make_float4(h2f_lo(vw[0]), h2f_hi(vw[0]), h2f_lo(vw[1]), h2f_hi(vw[1]));
-      vd[1] = make_float4(h2f_lo(vw[2]), h2f_hi(vw[2]), h2f_lo(vw[3]), h2f_hi(vw[3]));
-    }
-    if (n_old < nk) {  // new keys of this chunk (append): rotate from qkv, write the caches
-      for (int idx = n_old * kHeadDim + tid; idx < nk * kHeadDim; idx += kAttnThreads) {
-        const int j = idx / kHeadDim, d = idx - j * kHeadDim;
-        const int t = (int)(j0 + j - p0);
-        const __half* row = a.qkv + ((int64_t)b * T + t) * width;
-        const __half* kr = row + (int64_t)(a.Hq + kvh) * kHeadDim;
-        const __half vh = row[(int64_t)(a.Hq + a.Hkv + kvh) * kHeadDim + d];
-        const int pd = d & (kHeadDim / 2 - 1);
-        __half y1, y2;
-        rope_rotate_f16(__half2float(kr[pd]), __half2float(kr[pd + kHeadDim / 2]), cst[t * (kHeadDim / 2) + pd],
-                        y1, y2);
-        const __half kh = d < kHeadDim / 2 ? y1 : y2;
-        const int64_t off = hbase + j0 * kHeadDim + idx;
-        a.kcw[off] = kh;
-        a.vcw[off] = vh;
-        ks[j * kRowPad + d] = __half2float(kh);
-        vs[j * kRowPad + d] = __half2float(vh);
-      }
-    }
-    const int cn = c + S;
-    if (cn < nch) load_raw(cn);  // in flight while this chunk is computed
-    __syncthreads();
-    // scores: each thread a 2-query x 4-key tile
-    for (int tile = tid; tile < qpairs * (kAttnChunk / 4); tile += kAttnThreads) {
-      const int qp = tile / (kAttnChunk / 4), kq = tile - qp * (kAttnChunk / 4);
-      const int q0 = 2 * qp, q1 = q0 + 1 < Q ? q0 + 1 : q0;
-      float acc[2][4] = {};
-      const float4* qa = reinterpret_cast<const float4*>(qs + q0 * kRowPad);
-      const float4* qb = reinterpret_cast<const float4*>(qs + q1 * kRowPad);
-#pragma unroll 4
-      for (int d4 = 0; d4 < kHeadDim / 4; ++d4) {
-        const float4 x0 = qa[d4], x1 = qb[d4];
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-          const float4 kv = reinterpret_cast<const float4*>(ks + (4 * kq + kk) * kRowPad)[d4];
-          acc[0][kk] = fmaf(x0.x, kv.x, fmaf(x0.y, kv.y, fmaf(x0.z, kv.z, fmaf(x0.w, kv.w, acc[0][kk]))));
-          acc[1][kk] = fmaf(x1.x, kv.x, fmaf(x1.y, kv.y, fmaf(x1.z, kv.z, fmaf(x1.w, kv.w, acc[1][kk]))));
-        }
-      }
-#pragma unroll
-      for (int i = 0; i < 2; ++i) {
-        const int q = i ? q1 : q0;
-        if (i && q1 == q0) break;
-        const int t = q % T;
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-          const int j = 4 * kq + kk;
-          sc[q * kAttnChunk + j] = (j < nk && j0 + j <= (int64_t)p0 + t) ? acc[i][kk] : -INFINITY;
-        }
-      }
-    }
-    __syncthreads();
-    // online softmax update, one warp per query, one key per lane
-    const int warp = tid >> 5, lane = tid & 31;
-    for (int q = warp; q < Q; q += kAttnThreads / 32) {
-      const float v = sc[q * kAttnChunk + lane];
-      const float m_old = ms[q];
-      const float m_new = fmaxf(m_old, warp_max(v));
-      const float e = m_new == -INFINITY ? 0.0f : expf(v - m_new);
-      sc[q * kAttnChunk + lane] = e;
-      const float l = warp_sum(e);
-      if (lane == 0) {
-        const float alpha = m_old == -INFINITY ? 0.0f : expf(m_old - m_new);
-        al[q] = alpha;
-        ls[q] = fmaf(ls[q], alpha, l);
-        ms[q] = m_new;
-      }
-    }
-    __syncthreads();
-    // running weighted values: each thread a 2-query x 4-dim tile
-    for (int tile = tid; tile < qpairs * (kHeadDim / 4); tile += kAttnThreads) {
-      const int qp = tile / (kHeadDim / 4), d4 = tile - qp * (kHeadDim / 4);
-      const int q0 = 2 * qp, q1 = q0 + 1 < Q ? q0 + 1 : q0;
-      float4* p0v = reinterpret_cast<float4*>(os + q0 * kRowPad) + d4;
-      float4* p1v = reinterpret_cast<float4*>(os + q1 * kRowPad) + d4;
-      const float a0 = al[q0], a1 = al[q1];
-      float4 o0 = *p0v, o1 = *p1v;
-      o0.x *= a0; o0.y *= a0; o0.z *= a0; o0.w *= a0;
-      o1.x *= a1; o1.y *= a1; o1.z *= a1; o1.w *= a1;
-      for (int j = 0; j < nk; ++j) {
-        const float e0 = sc[q0 * kAttnChunk + j], e1 = sc[q1 * kAttnChunk + j];
-        const float4 vv = reinterpret_cast<const float4*>(vs + j * kRowPad)[d4];
-        o0.x = fmaf(e0, vv.x, o0.x); o0.y = fmaf(e0, vv.y, o0.y);
-        o0.z = fmaf(e0, vv.z, o0.z); o0.w = fmaf(e0, vv.w, o0.w);
-        o1.x = fmaf(e1, vv.x, o1.x); o1.y = fmaf(e1, vv.y, o1.y);
-        o1.z = fmaf(e1, vv.z, o1.z); o1.w = fmaf(e1, vv.w, o1.w);
-      }
-      *p0v = o0;
-      if (q1 != q0) *p1v = o1;
-    }
-    __syncthreads();
-    c = cn;
-  }
-
-  // merge the S states of this CTA's queries (q = rank, rank + S, ...)
-  attn_cluster_sync();
-  const int nq = (int)rank < Q ? (Q - 1 - (int)rank) / S + 1 : 0;
-  for (int idx = tid; idx < nq * kHeadDim; idx += kAttnThreads) {
-    const int q = (int)rank + (idx / kHeadDim) * S, d = idx - (idx / kHeadDim) * kHeadDim;
-    float mv[kClusterMaxS];
-    float M = -INFINITY;
-#pragma unroll
-    for (int r = 0; r < kClusterMaxS; ++r) {
-      mv[r] = r < S ? attn_ld_dsmem(ms + q, (uint32_t)r) : -INFINITY;
-      M = fmaxf(M, mv[r]);
-    }
-    float L = 0.0f, O = 0.0f;
-    if (M != -INFINITY) {
-#pragma unroll
-      for (int r = 0; r < kClusterMaxS; ++r) {
-        if (r >= S || mv[r] == -INFINITY) continue;
-        const float w = expf(mv[r] - M);
-        L = fmaf(w, attn_ld_dsmem(ls + q, (uint32_t)r), L);
-        O = fmaf(w, attn_ld_dsmem(os + q * kRowPad + d, (uint32_t)r), O);
-      }
-    }
-    const int g = q / T, t = q - g * T;
-    const int64_t row = (int64_t)b * T + t;
-    a.out[row * (int64_t)a.Hq * kHeadDim + (int64_t)(kvh * a.G + g) * kHeadDim + d] =
-        __float2half_rn(L > 0.0f ? O / L : 0.0f);
-  }
-  attn_cluster_sync();  // no CTA leaves while another still reads its state
-}
-
 // ---- embedding ---------------------------------------------------------------------
 // out[m, :] = table[ids[m], :] (fp16 copy, 16-byte pieces when aligned); an id
 // outside [0, V) gives a zero row and sets SQ_DEV_BAD_TOKEN_ID.
@@ -820,49 +540,6 @@ size_t attention_smem_bytes(int Q) {
 
 int attention_max_tokens() { return kMaxT; }
 
-// One cluster of S CTAs per (sequence, key/value head): S grows until about
-// two CTAs per SM are launched, at most the portable cluster size and the
-// number of cache chunks.
-static cudaError_t launch_attention_cluster(AttnArgs a, cudaStream_t st) {
-  const int groups = a.B * a.Hkv;
-  int S = (2 * device_sm_count() + groups - 1) / groups;
-  S = S < 1 ? 1 : (S > kClusterMaxS ? kClusterMaxS : S);
-  if (S > a.nsplit) S = a.nsplit;
-  a.S = S;
-  const size_t smem = attention_cluster_smem_bytes(a.T, a.Q);
-  static int smem_set[64] = {0};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if ((int)smem > smem_set[dev]) {
-    e = cudaFuncSetAttribute(attention_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    smem_set[dev] = (int)smem;
-  }
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)groups, (unsigned)S, 1);
-  cfg.blockDim = dim3(kAttnThreads);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[2];
-  int na = 0;
-  attr[na].id = cudaLaunchAttributeClusterDimension;
-  attr[na].val.clusterDim.x = 1;
-  attr[na].val.clusterDim.y = (unsigned)S;
-  attr[na].val.clusterDim.z = 1;
-  ++na;
-  const bool legacy = (st == nullptr || st == cudaStreamLegacy || st == cudaStreamPerThread);
-  if (!legacy && pdl_enabled()) {
-    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[na].val.programmaticStreamSerializationAllowed = 1;
-    ++na;
-  }
-  cfg.attrs = attr;
-  cfg.numAttrs = na;
-  return cudaLaunchKernelEx(&cfg, attention_cluster_kernel, a);
-}
-
 cudaError_t launch_attention(const __half* qkv, int B, int T, int Hq, int Hkv, const int32_t* pos0,
                              double theta, const __half* kc, const __half* vc, int64_t max_ctx,
                              __half* out, void* ws, cudaStream_t st, __half* kc_append,
@@ -888,7 +565,6 @@ cudaError_t launch_attention(const __half* qkv, int B, int T, int Hq, int Hkv, c
   a.nsplit = (int)((max_ctx + kAttnChunk - 1) / kAttnChunk);
   a.rf = rope_freq(theta);
   a.scale = 1.0f / sqrtf((float)kHeadDim);
-  if (a.Q <= kClusterMaxQ) return launch_attention_cluster(a, st);
   const size_t smem = attention_smem_bytes(a.Q);
   static int smem_set[64] = {0};
   int dev = 0;

@@ -46,10 +46,10 @@ def _fill_prefix(rng, B, Hkv, max_ctx, pos0):
     (2, 5, 12, 2, [37, 300], 512),
     (1, 1, 12, 2, [1023], 1024),
     (3, 9, 28, 4, [64, 127, 700], 1024),
-    (1, 17, 12, 2, [0], 64),            # 102 queries per group: chunk CTAs + combine kernel
-    (1, 1, 12, 2, [3000], 4096),        # a cluster CTA walks ~12 chunks (online softmax)
-    (2, 3, 12, 2, [5, 0], 128),         # fewer chunks than cluster CTAs; an empty prefix
-    (1, 32, 4, 2, [100], 256),          # 64 queries per group, the largest one-launch group
+    (1, 17, 12, 2, [0], 64),            # 102 queries per group
+    (1, 1, 12, 2, [3000], 4096),        # 94 chunks merged by the combine
+    (2, 3, 12, 2, [5, 0], 128),         # one chunk in use; an empty prefix
+    (1, 32, 4, 2, [100], 256),          # T at its limit
 ])
 def test_append_and_attention_match_oracle(B, T, Hq, Hkv, pos0, max_ctx):
     rng = np.random.default_rng(B * 100 + T)
