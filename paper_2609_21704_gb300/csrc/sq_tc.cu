@@ -166,6 +166,7 @@ struct TcArgs {
   int sc_ng;        // INT4: groups per row held in the block (>= any CTA's need)
   int max_split;    // largest split-K factor whose partial tile fits in the stages
   int two_per_sm;   // stages sized so that two CTAs share an SM
+  int int4_large;   // INT4 weights of 20 MB and more at few rows: power-of-two split rule
   const __half* bias;
   const __half* residual;
   __half* y;
@@ -587,7 +588,18 @@ static int tc_max_clusters(int S, size_t smem) {
 // CTA + 2 for the split reduction), at least 2 k-steps per CTA; ties keep
 // the smaller S.
 template <int WK, bool SILU>
-static int tc_pick_split(int64_t tiles, int ksteps, size_t smem, int max_split, bool two_per_sm) {
+static int tc_pick_split(int64_t tiles, int ksteps, size_t smem, int max_split, bool two_per_sm,
+                         bool int4_large = false) {
+  if (WK == 1 && int4_large) {
+    // two CTAs per SM: the largest power-of-two split with at most 2.2 CTAs
+    // per SM in all and at least 12 k-steps per CTA (odd splits of 3 and 7
+    // measured 20-50 % slower than their neighbours)
+    const int sms = device_sm_count();
+    int S = 1;
+    for (int s = 2; s <= max_split && s <= kTcMaxSplitInt4; s <<= 1)
+      if (tiles * s * 10 <= 22 * (int64_t)sms && ksteps >= 12 * s) S = s;
+    return S;
+  }
   if (WK != 1) {
     const int sms = device_sm_count();
     int S = 1;
@@ -623,7 +635,8 @@ static cudaError_t tc_launch_inst(const CUtensorMap& tw, const CUtensorMap& tx, 
   auto k = tc_linear_kernel<WK, SILU>;
   cudaError_t e = tc_prepare<WK, SILU>(smem);
   if (e != cudaSuccess) return e;
-  const int S = tc_pick_split<WK, SILU>(tiles, a.ksteps, smem, a.max_split, a.two_per_sm != 0);
+  const int S = tc_pick_split<WK, SILU>(tiles, a.ksteps, smem, a.max_split, a.two_per_sm != 0,
+                                       a.int4_large != 0);
   a.splits = S;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)S, (unsigned)tiles, 1);
@@ -714,8 +727,15 @@ cudaError_t launch_tc(int wk, const __half* x, const void* w, const void* scales
   // CTA's prologue and epilogue overlap the other's loads (measured 8-28 %
   // faster on the 1.5B/7B down, qkv and o shapes); otherwise one CTA per SM
   // with 200 KB of stages.
+  // INT4 weights of 20 MB and more at NB <= 64 (the draft pass at 8 or 16
+  // rows: 7B/14B gate/up, down and lm_head) take two CTAs per SM too, with a
+  // power-of-two split: measured 20-40 % faster than one CTA per SM with the
+  // occupancy cost model (14B lm_head at M = 16: 332 -> 203 us; gate/up 57
+  // -> 45 us; down 45 -> 36 us).
   const int sms = device_sm_count();
-  a.two_per_sm = (nb <= 64 && tiles * 2 <= sms) ? 1 : 0;
+  const double wbytes = (double)wrows * (double)(K / 2) + (double)wrows * (double)(K / 128) * 2.0;
+  a.int4_large = (wk == SQ_W_INT4 && nb <= 64 && wbytes >= 20e6) ? 1 : 0;
+  a.two_per_sm = (a.int4_large || (nb <= 64 && tiles * 2 <= sms)) ? 1 : 0;
   const int budget = (a.two_per_sm ? 100 : 200) * 1024;
   int ns = (int)((budget - (int64_t)sc_bytes) / a.stage_bytes);
   if (ns > 8) ns = 8;

@@ -199,3 +199,29 @@ def test_tc_silu_largest_m(kind):
     assert sq.sq_check() == 0
     full = oracle.linear(x.astype(np.float64), w64)
     assert_close(dev_to_f64(y), oracle.silu_gate(full[:, :I], full[:, I:]), f"{kind} silu M=256")
+
+
+@pytest.mark.parametrize("M,N,K,epi", [
+    (16, 8192, 5120, sq.SQ_EPI_NONE),         # 21.5 MB of INT4: two CTAs per SM, split 4
+    (8, 5120, 13824, sq.SQ_EPI_NONE),         # the 14B down shape: split 8
+    (16, 2 * 6912, 5120, sq.SQ_EPI_SILU_GATE),  # a fused gate/up of 36 MB: split 2
+])
+def test_tc_int4_large_matrices_sampled(M, N, K, epi):
+    # INT4 matrices of 20 MB and more at few rows take their own split rule;
+    # checked on sampled output columns (the oracle dequantises those rows)
+    w = synth.weights_fp16(N + K + M, N, K)
+    x = synth.activations_fp16(M + 3, M, K)
+    c, s = oracle.quantize_int4(w.view(np.uint16))
+    y = torch.empty(M, N // 2 if epi == sq.SQ_EPI_SILU_GATE else N, dtype=torch.float16, device=dev())
+    assert sq.sq_linear_path(sq.SQ_W_INT4, M, y.shape[1], K, epi) == 1
+    sq.sq_linear_ex(sq.SQ_W_INT4, f16_to_dev(x), torch.from_numpy(c).to(dev()), f16_to_dev(s.view(np.float16)),
+                    None, None, epi, y)
+    assert sq.sq_check() == 0
+    ncol = y.shape[1]
+    cols = np.unique(np.concatenate([[0, ncol - 1], np.random.default_rng(M).integers(0, ncol, 62)]))
+    rows = cols if epi != sq.SQ_EPI_SILU_GATE else np.concatenate([cols, cols + ncol])
+    w64 = oracle.dequant_int4(c[rows], s[rows], K)
+    ref = oracle.linear(x.astype(np.float64), w64)
+    if epi == sq.SQ_EPI_SILU_GATE:
+        ref = oracle.silu_gate(ref[:, :len(cols)], ref[:, len(cols):])
+    assert_close(dev_to_f64(y)[:, cols], ref, f"int4 M={M} N={N} K={K}")
