@@ -193,7 +193,9 @@ _COMMON = ("sq_device.cuh", "sq_internal.h", "sq_plan.cu")
 
 def kernel_digest(kernel_tag: str) -> str:
     engine, fmt = kernel_tag.split("_")[:2]
-    files = (("sq_gemv.cuh", f"sq_gemv_{fmt}.cu") if engine == "gemv" else ("sq_tc.cu",)) + _COMMON
+    files = {"gemv": ("sq_gemv.cuh", f"sq_gemv_{fmt}.cu"),
+             "mma": ("sq_gemv.cuh", "sq_gemv_mma.cuh", f"sq_gemv_{fmt}.cu"),
+             "tc": ("sq_tc.cu",)}[engine] + _COMMON
     return source_digest([os.path.join(_CSRC, f) for f in files])
 
 
@@ -539,8 +541,8 @@ def main():
 
     # ---- dominant kernel: the fused gate/up + SiLU linear (largest per-launch
     # weight matrix in the layers); all layers' launches of it in one graph
-    engine = "tc" if sq.sq_linear_path(stk.WKIND[args.draft], B, shape.intermediate, shape.hidden,
-                                       sq.SQ_EPI_SILU_GATE) == 1 else "gemv"
+    engine = {1: "tc", 2: "mma"}.get(sq.sq_linear_path(stk.WKIND[args.draft], B, shape.intermediate,
+                                                      shape.hidden, sq.SQ_EPI_SILU_GATE), "gemv")
     kernel_tag = f"{engine}_{args.draft}_gateup_silu_m{B}"
     gu_projs = [layer[2] for layer in stack.layers]
 

@@ -124,11 +124,13 @@ SQ_API sq_status sq_quantize(const void* w16, int64_t N, int64_t K, sq_qkind kin
  * fp16 [N] or NULL.  Products are exact and sums are fp32; y is rounded to
  * nearest fp16 once.  1 <= M <= 256; N >= 1; K as for sq_quantize (INT4:
  * K % 128 == 0, FP8: K % 16 == 0, FP16: K % 8 == 0).  x, codes, w16 and y
- * must be 16-byte aligned.  Each call runs on one of two engines, chosen
+ * must be 16-byte aligned.  Each call runs on one of these engines, chosen
  * from (format, M, N, K, epilogue) alone (sq_linear_path reports which):
- * the CUDA-core GEMV family for few rows, the tcgen05 tensor-core tile path
- * from 16 rows on and, below that, for the formats and shapes where it is
- * faster.  Both give the same fp32-accumulated result up to summation order.
+ * the CUDA-core GEMV family for few rows (for one INT4 row over many output
+ * rows, with its products on the tensor cores' register-operand path), the
+ * tcgen05 tensor-core tile path from 16 rows on and, below that, for the
+ * formats and shapes where it is faster.  All give the same fp32-accumulated
+ * result up to summation order.
  * y must not overlap x, the weights or the scales.
  * ---------------------------------------------------------------------- */
 SQ_API sq_status sq_linear_w4a16(const void* x, const void* codes, const void* scales,
@@ -171,8 +173,10 @@ SQ_API sq_status sq_linear_norm(sq_wkind wkind, const void* x, const void* gamma
                                 sq_epilogue epi, void* y, int M, int64_t N, int64_t K, sq_stream_t stream);
 
 /* Engine sq_linear_ex would use for these sizes: 1 = tcgen05 tensor cores,
- * 0 = CUDA-core GEMV, -1 = sizes or kinds sq_linear_ex rejects (pointers are
- * not examined; nothing runs on the device).  The paper has no counterpart:
+ * 0 = CUDA-core GEMV, 2 = one INT4 activation row over at least 304 16-row
+ * output tiles with the products on the tensor cores' register-operand path
+ * (mma.sync), -1 = sizes or kinds sq_linear_ex rejects (pointers are not
+ * examined; nothing runs on the device).  The paper has no counterpart:
  * this is introspection for tests and tuning. */
 SQ_API int sq_linear_path(sq_wkind wkind, int M, int64_t N, int64_t K, sq_epilogue epi);
 

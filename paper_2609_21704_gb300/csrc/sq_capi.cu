@@ -153,8 +153,9 @@ static sq_status check_linear(const sq_linear_op& op) {
 }
 
 // Launches one checked call.
-// gamma != null: y = linear(rmsnorm(x) * gamma).  The GEMV normalises the rows
-// it stages; the tensor-core path writes the normalised rows to xn first.
+// gamma != null: y = linear(rmsnorm(x) * gamma).  The GEMV kernels normalise
+// the rows they stage; the tensor-core tile path writes the normalised rows to
+// xn first.
 static sq_status run_linear(const sq_linear_op& op, cudaStream_t stream, const __half* gamma = nullptr,
                             float eps = 0.0f, __half* xn = nullptr) {
   GemvArgs a = {};
@@ -174,13 +175,16 @@ static sq_status run_linear(const sq_linear_op& op, cudaStream_t stream, const _
   a.pieces = (int)(op.K / weights_per_piece(op.wkind));
   a.ppad = (a.pieces + 31) / 32 * 32;
   cudaError_t e;
-  if (use_tensor_cores(op.wkind, op.M, op.N, op.K, op.epi) && tc_supported(op.M, op.K, op.epi)) {
+  const bool tc = use_tensor_cores(op.wkind, op.M, op.N, op.K, op.epi) && tc_supported(op.M, op.K, op.epi);
+  if (gamma && tc) {
+    // the tensor-core tile path stages x by TMA: the standalone RMSNorm first
+    e = launch_rmsnorm(a.x, gamma, op.M, op.K, eps, xn, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "sq_linear_norm: rmsnorm launch");
+    a.x = xn;
+    a.gamma = nullptr;
+  }
+  if (tc) {
     // tcgen05 tensor cores, weights on the MMA's M side
-    if (gamma) {
-      e = launch_rmsnorm(a.x, gamma, op.M, op.K, eps, xn, stream);
-      if (e != cudaSuccess) return cuda_fail(e, "sq_linear_norm: rmsnorm launch");
-      a.x = xn;
-    }
     e = launch_tc(op.wkind, a.x, op.w, op.scales, a.bias, a.residual, a.y, op.M, op.N, op.K, op.epi,
                   stream);
     if (e != cudaSuccess) return cuda_fail(e, "sq_linear: tensor-core launch");
@@ -255,7 +259,8 @@ sq_status sq_linear_chain(const sq_linear_op* ops, int count, sq_stream_t stream
 
 int sq_linear_path(sq_wkind wkind, int M, int64_t N, int64_t K, sq_epilogue epi) {
   if (check_linear_sizes(wkind, M, N, K, epi) != SQ_OK) return -1;
-  return use_tensor_cores(wkind, M, N, K, epi) && tc_supported(M, K, epi) ? 1 : 0;
+  if (use_tensor_cores(wkind, M, N, K, epi) && tc_supported(M, K, epi)) return 1;
+  return gemv_uses_mma(wkind, M, N) ? 2 : 0;
 }
 
 sq_status sq_linear_w4a16(const void* x, const void* codes, const void* scales, const void* bias,

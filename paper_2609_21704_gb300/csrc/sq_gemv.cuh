@@ -106,6 +106,21 @@ __device__ __forceinline__ float dot8_natural(uint32_t w0, uint32_t w1, uint32_t
   return acc;
 }
 
+// Output (row m, column n) from its fp32 dot product v (and, with the SiLU
+// gate, the up row's u): FP8 row scale, bias, silu(v) * u, residual, fp16.
+template <int WK, bool SILU>
+__device__ __forceinline__ void gemv_store(const GemvArgs& a, int64_t n, int m, float v, float u) {
+  if constexpr (WK == WK_FP8) v *= reinterpret_cast<const float*>(a.scales)[n];
+  if (a.bias) v += __half2float(a.bias[n]);
+  if constexpr (SILU) {
+    if constexpr (WK == WK_FP8) u *= reinterpret_cast<const float*>(a.scales)[a.N + n];
+    if (a.bias) u += __half2float(a.bias[a.N + n]);
+    v = v / (1.0f + expf(-v)) * u;
+  }
+  if (a.residual) v += __half2float(a.residual[(int64_t)m * a.N + n]);
+  a.y[(int64_t)m * a.N + n] = __float2half_rn(v);
+}
+
 // Pieces of one weight row a lane keeps in flight per batch: enough bytes
 // in flight to cover DRAM latency (U x 512 B per row per warp) within the
 // register budget.
@@ -403,17 +418,9 @@ __global__ void __launch_bounds__(kGemvThreads, (GemvMinBlocks<WK, MR, R, SILU>:
 #pragma unroll
       for (int m = 0; m < MR; ++m) {
         if (m >= a.M || ll != ((r * MR + m) % LPR)) continue;
-        float v = acc[r][m];
-        if constexpr (WK == WK_FP8) v *= reinterpret_cast<const float*>(a.scales)[n];
-        if (a.bias) v += __half2float(a.bias[n]);
-        if constexpr (SILU) {
-          float u = acc[R + r][m];
-          if constexpr (WK == WK_FP8) u *= reinterpret_cast<const float*>(a.scales)[a.N + n];
-          if (a.bias) u += __half2float(a.bias[a.N + n]);
-          v = v / (1.0f + expf(-v)) * u;
-        }
-        if (a.residual) v += __half2float(a.residual[(int64_t)m * a.N + n]);
-        a.y[(int64_t)m * a.N + n] = __float2half_rn(v);
+        float u = 0.0f;
+        if constexpr (SILU) u = acc[R + r][m];
+        gemv_store<WK, SILU>(a, n, m, acc[r][m], u);
       }
     }
   }

@@ -99,6 +99,9 @@ bool use_tensor_cores(int wk, int M, int64_t N, int64_t K, int epi) {
 }
 
 cudaError_t launch_gemv(int wk, const GemvArgs& a0, cudaStream_t st) {
+  // one INT4 row over many 16-row tiles: products on the tensor cores
+  if (gemv_uses_mma(wk, a0.M, a0.N))
+    return launch_gemv_mma_int4(a0, a0.epi == SQ_EPI_SILU_GATE, st);
   GemvArgs a = a0;
   const int cap = gemv_cap_mr(wk, a.K);
   if (cap == 0) return cudaErrorInvalidValue;

@@ -182,3 +182,36 @@ def test_full_size_down_proj_7b(kind, M):
 @pytest.mark.parametrize("kind,M", [("int4", 1), ("fp16", 5)])
 def test_full_size_gate_up_silu_7b(kind, M):
     _sampled_full_size(kind, QWEN25_7B.projections()[2], M, epi=sq.SQ_EPI_SILU_GATE, seed=5)
+
+
+# ---- INT4 single-row calls with many 16-row tiles (the fused gate/up, the
+# lm_head) take the tensor cores' register path (mma.sync): every output
+# column of whole matrices, ragged tile counts, odd group counts, split K.
+@pytest.mark.parametrize("N,K,epi", [
+    (8960, 1536, sq.SQ_EPI_SILU_GATE),   # the 1.5B fused gate/up, whole
+    (4869, 896, sq.SQ_EPI_NONE),         # ragged last tile, 7 groups split 4 ways
+    (5003, 8960, sq.SQ_EPI_RESIDUAL),    # 70 groups, bias and residual
+    (40000, 256, sq.SQ_EPI_NONE),        # two groups, no split
+])
+def test_int4_single_row_tensor_path(N, K, epi):
+    Nw = 2 * N if epi == sq.SQ_EPI_SILU_GATE else N
+    assert sq.sq_linear_path(sq.SQ_W_INT4, 1, N, K, epi) == 2
+    w = synth.weights_fp16(Nw + 3 * K, Nw, K)
+    x = synth.activations_fp16(N + 7, 1, K)
+    b = synth.fp16_normal(Nw + 1, (Nw,), 1.0)
+    wd, sd, w64 = _variant("int4", w)
+    ref = oracle.linear(x.astype(np.float64), w64, b.astype(np.float64))
+    if epi == sq.SQ_EPI_RESIDUAL:
+        r = synth.fp16_normal(K + 1, (1, N), 1.0)
+        y = f16_to_dev(r)
+        _run("int4", f16_to_dev(x), wd, sd, N, bias=f16_to_dev(b), residual=y, epi=epi, y=y)
+        ref = ref + r.astype(np.float64)
+    else:
+        y = _run("int4", f16_to_dev(x), wd, sd, N, bias=f16_to_dev(b), epi=epi)
+        if epi == sq.SQ_EPI_SILU_GATE:
+            ref = oracle.silu_gate(ref[:, :N], ref[:, N:])
+    assert_close(dev_to_f64(y), ref, f"int4 tensor path N={N} K={K} epi={epi}")
+    y2 = _run("int4", f16_to_dev(x), wd, sd, N, bias=f16_to_dev(b), epi=epi) if epi != sq.SQ_EPI_RESIDUAL else None
+    if y2 is not None:
+        assert torch.equal(y, y2), "not repeatable bit for bit"
+    assert sq.sq_check() == 0

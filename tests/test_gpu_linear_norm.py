@@ -36,6 +36,7 @@ def _weights(kind, N, K, seed):
 @pytest.mark.parametrize("M,N,K,epi", [
     (1, 2048, 1536, sq.SQ_EPI_NONE),          # q/k/v of the 1.5B shape
     (1, 17920, 1536, sq.SQ_EPI_SILU_GATE),    # gate/up
+    (1, 9000, 896, sq.SQ_EPI_NONE),           # INT4: many 16-row tiles, register-operand tensor path
     (2, 640, 896, sq.SQ_EPI_NONE),
     (5, 2048, 1536, sq.SQ_EPI_NONE),          # verify rows
     (16, 1024, 3584, sq.SQ_EPI_SILU_GATE),

@@ -167,8 +167,12 @@ def test_tc_small_m_matches_oracle(kind, M, N, K, epi):
 
 
 def test_engine_choice_small_rows():
-    # few rows and small matrices stay on the CUDA-core GEMV
-    assert sq.sq_linear_path(sq.SQ_W_INT4, 1, 151936, 1536, sq.SQ_EPI_NONE) == 0
+    # few rows and small matrices stay on the CUDA-core GEMV; one INT4 row
+    # over many 16-row tiles takes the register-operand tensor-core path
+    assert sq.sq_linear_path(sq.SQ_W_INT4, 1, 151936, 1536, sq.SQ_EPI_NONE) == 2
+    assert sq.sq_linear_path(sq.SQ_W_INT4, 1, 8960, 1536, sq.SQ_EPI_SILU_GATE) == 2
+    assert sq.sq_linear_path(sq.SQ_W_INT4, 1, 2048, 1536, sq.SQ_EPI_NONE) == 0
+    assert sq.sq_linear_path(sq.SQ_W_FP8, 1, 151936, 1536, sq.SQ_EPI_NONE) == 0
     assert sq.sq_linear_path(sq.SQ_W_FP16, 5, 2048, 1536, sq.SQ_EPI_NONE) == 0
     assert sq.sq_linear_path(sq.SQ_W_FP16, 5, 151936, 1536, sq.SQ_EPI_NONE) == 0
     assert sq.sq_linear_path(sq.SQ_W_FP8, 5, 17920, 1536, sq.SQ_EPI_NONE) == 0
