@@ -31,7 +31,15 @@ from . import (SQ_ACCEPT_GREEDY, SQ_ACCEPT_SAMPLE, sq_accept_logits, sq_accept_l
                sq_check, sq_embed, sq_sample_logits, sq_spec_commit, sq_spec_drafts, synth)
 from .stack import DecoderState, LinearStack, decoder_pass
 
-PREFILL_CHUNK = 32   # tokens per prefill pass (the attention kernel's T limit)
+# Limits of one sq_attention call (see its declaration): at most 32 new
+# tokens per sequence, and (Hq / Hkv) * T <= 200 queries per key/value head.
+ATTN_MAX_T = 32
+ATTN_MAX_GROUP_QUERIES = 200
+
+
+def prefill_chunk(q_heads: int, kv_heads: int) -> int:
+    """Tokens per prefill pass: as many as one attention call takes."""
+    return min(ATTN_MAX_T, ATTN_MAX_GROUP_QUERIES // (q_heads // kv_heads))
 
 
 class Generator:
@@ -64,7 +72,8 @@ class Generator:
             self.d2 = DecoderState(stack, B, 2, max_ctx, share_gains=self.tv)
             if K > 1:
                 self.d1 = DecoderState(stack, B, 1, max_ctx, share=self.d2)
-        self.chunks = [(s, min(PREFILL_CHUNK, prompt_len - s)) for s in range(0, prompt_len, PREFILL_CHUNK)]
+        pc = prefill_chunk(sh.q_heads, sh.kv_heads)
+        self.chunks = [(s, min(pc, prompt_len - s)) for s in range(0, prompt_len, pc)]
         self.pre_t, self.pre_d = {}, {}
         for _, T in self.chunks:
             if T not in self.pre_t:
