@@ -116,3 +116,23 @@ def test_accept_validation(lib):
 def test_binding_fails_loudly_without_the_library(tmp_path):
     with pytest.raises(ImportError):
         sq.load(str(tmp_path / "missing.so"))
+
+
+def test_single_row_engine_choice(lib):
+    """sq_linear_path is host logic: one INT4 activation row over at least 304
+    16-row output tiles takes the register-operand tensor path (2), other
+    single-row calls the streaming CUDA-core GEMV (0)."""
+    W4, W8, W16 = sq.SQ_W_INT4, sq.SQ_W_FP8, sq.SQ_W_FP16
+    NONE, SILU, RES = sq.SQ_EPI_NONE, sq.SQ_EPI_SILU_GATE, sq.SQ_EPI_RESIDUAL
+    assert sq.sq_linear_path(W4, 1, 8960, 1536, SILU) == 2      # 1.5B fused gate/up
+    assert sq.sq_linear_path(W4, 1, 151936, 1536, NONE) == 2    # 1.5B lm_head
+    assert sq.sq_linear_path(W4, 1, 18944, 3584, SILU) == 2     # 7B fused gate/up
+    assert sq.sq_linear_path(W4, 1, 2048, 1536, NONE) == 0      # 1.5B q/k/v
+    assert sq.sq_linear_path(W4, 1, 1536, 1536, RES) == 0       # 1.5B o
+    assert sq.sq_linear_path(W4, 1, 1536, 8960, RES) == 0       # 1.5B down
+    assert sq.sq_linear_path(W4, 1, 16 * 304, 896, NONE) == 2   # exactly 304 tiles
+    assert sq.sq_linear_path(W4, 1, 16 * 304 - 16, 896, NONE) == 0
+    assert sq.sq_linear_path(W4, 1, 16 * 303 + 1, 896, NONE) == 2  # ragged 304th tile
+    assert sq.sq_linear_path(W4, 2, 151936, 1536, NONE) == 0    # two rows: streaming GEMV
+    assert sq.sq_linear_path(W8, 1, 151936, 1536, NONE) == 0
+    assert sq.sq_linear_path(W16, 1, 151936, 1536, NONE) == 0
