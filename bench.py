@@ -255,19 +255,19 @@ def cpu_oracle_prepare(shape, variant, B, K, layers=1, lm_rows=None, seed=0):
             "zp": zp, "zq": zq, "u_draft": u_draft}
 
 
-def cpu_oracle_run(prep, draft, u):
-    """One timed oracle step on the prepared sample; returns (seconds of
-    the full step extrapolated by weight count, seconds spent)."""
+def _oracle_linears(items, variant, K):
+    """Seconds the oracle spends on the linear part of one step over `items`:
+    dequantise each matrix, K draft linears, one verify linear."""
     import oracle
 
     t_lin = 0.0
-    for n, k, silu, w16, (codes, sc), xd, xv in prep["items"]:
+    for n, k, silu, w16, (codes, sc), xd, xv in items:
         t0 = time.perf_counter()
-        if prep["variant"] == "int4":
+        if variant == "int4":
             wq = oracle.dequant_int4(codes, sc, k)
         else:
             wq = oracle.dequant_fp8(codes, sc)
-        for _ in range(prep["K"]):
+        for _ in range(K):
             yd = oracle.linear(xd, wq)
             if silu:
                 oracle.silu_gate(yd[:, : n // 2], yd[:, n // 2:])
@@ -275,12 +275,90 @@ def cpu_oracle_run(prep, draft, u):
         if silu:
             oracle.silu_gate(yv[:, : n // 2], yv[:, n // 2:])
         t_lin += time.perf_counter() - t0
+    return t_lin
+
+
+def cpu_oracle_run(prep, draft, u):
+    """One timed oracle step on the prepared sample; returns (seconds of
+    the full step extrapolated by weight count, seconds spent, seconds of
+    the draft samples and the accept)."""
+    import oracle
+
+    t_lin = _oracle_linears(prep["items"], prep["variant"], prep["K"])
     t0 = time.perf_counter()
     for k in range(prep["K"]):
         oracle.sample_logits(prep["zq"][k], prep["u_draft"][k])
     oracle.accept_logits(prep["zp"], prep["zq"], draft, u, 1.0, oracle.ACCEPT_SAMPLE)
     t_acc = time.perf_counter() - t0
-    return t_lin * prep["scale"] + t_acc, t_lin + t_acc
+    return t_lin * prep["scale"] + t_acc, t_lin + t_acc, t_acc
+
+
+def _row_slice(item, w, P):
+    """Output-row slice w of P of one sample matrix (gate and up rows together
+    for the fused gate/up)."""
+    import numpy as np
+
+    n, k, silu, w16, (codes, sc), xd, xv = item
+    if silu:
+        half = n // 2
+        a, b = w * half // P, (w + 1) * half // P
+        rows = np.r_[a:b, half + a:half + b]
+    else:
+        a, b = w * n // P, (w + 1) * n // P
+        rows = np.arange(a, b)
+    return (len(rows), k, silu, w16[rows], (codes[rows], sc[rows]), xd, xv)
+
+
+def _cpu_all_cores_worker(w, P, workload, variant, B, K, reps, barrier, results):
+    """One process of the all-cores oracle baseline: the same sample as the
+    single-thread run, its output-row slice w of P of every matrix, timed
+    `reps` times, each start aligned with the other processes by `barrier`."""
+    from paper_2609_21704_gb300.shapes import STACKS
+
+    prep = cpu_oracle_prepare(STACKS[workload], variant, B, K, layers=1)
+    items = [_row_slice(it, w, P) for it in prep["items"]]
+    items = [it for it in items if it[0] > 0]
+    for r in range(reps):
+        barrier.wait(timeout=120)
+        results.put((w, r, _oracle_linears(items, variant, K)))
+
+
+def cpu_oracle_all_cores(shape, variant, B, K, scale, t_accept, tokens_per_step, reps=3):
+    """The oracle as it stands, on every host core: one spawned process per
+    core, each running the single-thread sample's linear part on its slice of
+    output rows; a step's linear time is the slowest process's, extrapolated
+    by weight count like the single-thread run; the accept part is the
+    single-thread run's (it is not split)."""
+    import multiprocessing as mp
+
+    P = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+    ctx = mp.get_context("spawn")
+    barrier, results = ctx.Barrier(P), ctx.Queue()
+    procs = [ctx.Process(target=_cpu_all_cores_worker,
+                         args=(w, P, shape.name, variant, B, K, reps, barrier, results), daemon=True)
+             for w in range(P)]
+    for p in procs:
+        p.start()
+    deadline = time.monotonic() + 120.0  # the whole leg, so a dead worker cannot stall the bench
+    try:
+        per_rep = {}
+        for _ in range(P * reps):
+            w, r, t = results.get(timeout=max(1.0, deadline - time.monotonic()))
+            per_rep[r] = max(per_rep.get(r, 0.0), t)
+    finally:
+        for p in procs:
+            p.join(timeout=30)
+            if p.is_alive():
+                p.terminate()
+    t_lin = statistics.median(per_rep.values())
+    t_full = t_lin * scale + t_accept
+    return {"value": tokens_per_step / t_full, "unit": UNIT, "cores": P, "kind": "oracle",
+            "sample": (f"the single-thread sample's linear part split by output rows over {P} "
+                       f"spawned processes (one per host core), slowest process per step, "
+                       f"median of {reps}; the draft samples and the accept single-threaded; "
+                       f"row slices alone run the oracle's linears faster per weight than whole "
+                       f"matrices (its fp64 temporaries), so the ratio to the 1-core figure can "
+                       f"exceed the core count")}
 
 
 # ----------------------------------------------------------------------------- main
@@ -603,7 +681,7 @@ def main():
                "ms_per_step": 1e3 * t_e2e / e2e_steps, "steps": e2e_steps}
 
     # ---- CPU oracle baseline (rank 0, N = 1)
-    cpu = None
+    cpu = cpu_all = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         prep = cpu_oracle_prepare(shape, args.draft, B, K, layers=1)
         runs = [cpu_oracle_run(prep, draft, u) for _ in range(3)]
@@ -611,6 +689,12 @@ def main():
         cpu = {"value": tokens_per_step / t_full, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": prep["desc"] + "; median of 3 runs",
                "sample_seconds": round(sum(r[1] for r in runs), 2)}
+        # the same oracle on every host core (a second baseline, not the target)
+        try:
+            cpu_all = cpu_oracle_all_cores(shape, args.draft, B, K, prep["scale"],
+                                           statistics.median(r[2] for r in runs), tokens_per_step)
+        except Exception as exc:  # a failed baseline must not cost the bench line
+            cpu_all = {"error": f"{type(exc).__name__}: {exc}"}
 
     if rank != 0:
         return 0
@@ -677,6 +761,7 @@ def main():
                      "algorithmic_bytes_per_launch": gu_bytes, "avg_launch_us": 1e6 * t_gu,
                      "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs, copy)"},
         "cpu_baseline": cpu,
+        "cpu_baseline_all_cores": cpu_all,
         "e2e": e2e,
         "clocks": clk,
         "gpu_launches": launches_per_step * args.steps,
@@ -756,7 +841,7 @@ def main_reference():
     desc = prep["desc"]
     times = []
     for i in range(args.warmup + args.steps):
-        t_full, _ = cpu_oracle_run(prep, draft, u)
+        t_full = cpu_oracle_run(prep, draft, u)[0]
         if i >= args.warmup:
             times.append(t_full)
     t = sum(times)
