@@ -145,7 +145,9 @@ def sq_version() -> int:
 
 
 def sq_linear_path(wkind: int, M: int, N: int, K: int, epi: int = SQ_EPI_NONE) -> int:
-    """1: tensor cores, 0: CUDA-core GEMV, -1: sizes sq_linear_ex rejects."""
+    """1: tcgen05 tensor-core tiles, 0: CUDA-core GEMV, 2: one INT4 row with
+    its products on the tensor cores' register-operand path, -1: sizes
+    sq_linear_ex rejects."""
     return load().sq_linear_path(wkind, M, N, K, epi)
 
 
