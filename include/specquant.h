@@ -165,8 +165,9 @@ SQ_API sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, cons
  * sq_rmsnorm's (fp32 arithmetic, the normalised rows rounded to fp16) and
  * the result is bit-identical to sq_rmsnorm followed by sq_linear_ex.  The
  * CUDA-core GEMV normalises the activation rows as it stages them (no extra
- * launch); the tensor-core path writes them to xn (fp16 [M, K], 16-byte
- * aligned, not aliasing x, y or the residual) first.  gamma fp16 [K], 16-byte
+ * launch); the tensor-core path and the shared-memory ring engine write them
+ * to xn (fp16 [M, K], 16-byte aligned, not aliasing x, y or the residual)
+ * first.  gamma fp16 [K], 16-byte
  * aligned; eps >= 0. */
 SQ_API sq_status sq_linear_norm(sq_wkind wkind, const void* x, const void* gamma, float eps, void* xn,
                                 const void* w, const void* scales, const void* bias, const void* residual,
@@ -175,9 +176,11 @@ SQ_API sq_status sq_linear_norm(sq_wkind wkind, const void* x, const void* gamma
 /* Engine sq_linear_ex would use for these sizes: 1 = tcgen05 tensor cores,
  * 0 = CUDA-core GEMV, 2 = one INT4 activation row over at least 304 16-row
  * output tiles with the products on the tensor cores' register-operand path
- * (mma.sync), -1 = sizes or kinds sq_linear_ex rejects (pointers are not
- * examined; nothing runs on the device).  The paper has no counterpart:
- * this is introspection for tests and tuning. */
+ * (mma.sync), 3 = one activation row streamed through a shared-memory ring
+ * of asynchronous copies, products on the same register-operand path,
+ * -1 = sizes or kinds sq_linear_ex rejects (pointers are not examined;
+ * nothing runs on the device).  The paper has no counterpart: this is
+ * introspection for tests and tuning. */
 SQ_API int sq_linear_path(sq_wkind wkind, int M, int64_t N, int64_t K, sq_epilogue epi);
 
 /* Sec. III-D.2 / III-D.3: a draft or verify pass runs every projection of
@@ -202,6 +205,7 @@ typedef struct sq_linear_op {
   void* y;               /* fp16 [M, N] */
 } sq_linear_op;
 SQ_API sq_status sq_linear_chain(const sq_linear_op* ops, int count, sq_stream_t stream);
+
 
 /* ------------------------------------------------------------------------
  * Sec. III-A.3 token rule and Sec. III-D.4 acceptance / correction, for a

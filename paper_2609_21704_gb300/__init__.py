@@ -146,8 +146,8 @@ def sq_version() -> int:
 
 def sq_linear_path(wkind: int, M: int, N: int, K: int, epi: int = SQ_EPI_NONE) -> int:
     """1: tcgen05 tensor-core tiles, 0: CUDA-core GEMV, 2: one INT4 row with
-    its products on the tensor cores' register-operand path, -1: sizes
-    sq_linear_ex rejects."""
+    its products on the tensor cores' register-operand path, 3: one row
+    through the shared-memory ring engine, -1: sizes sq_linear_ex rejects."""
     return load().sq_linear_path(wkind, M, N, K, epi)
 
 
@@ -191,12 +191,17 @@ class SqLinearOp(ctypes.Structure):
 def sq_linear_chain(ops, stream=None) -> None:
     """ops: sequence of (wkind, x, w, scales, bias, residual, epi, y) with the
     same meaning as sq_linear_ex's arguments; run in order (one C call)."""
+    arr = _op_array(ops)
+    _check("sq_linear_chain", load().sq_linear_chain(ctypes.cast(arr, _P), len(ops), _stream(stream)))
+
+
+def _op_array(ops):
     arr = (SqLinearOp * max(1, len(ops)))()
     for i, (wkind, x, w, scales, bias, residual, epi, y) in enumerate(ops):
         M, K = x.shape
         arr[i] = SqLinearOp(wkind, epi, M, 0, y.shape[1], K, _ptr(x), _ptr(w), _ptr(scales),
                             _ptr(bias), _ptr(residual), _ptr(y))
-    _check("sq_linear_chain", load().sq_linear_chain(ctypes.cast(arr, _P), len(ops), _stream(stream)))
+    return arr
 
 
 def sq_linear_w4a16(x, codes, scales, bias, y, stream=None) -> None:

@@ -64,7 +64,7 @@ sq_status sq_check(sq_stream_t stream, uint32_t* device_bits) {
   if ((e = take_gemv_status_int4(&bits)) != cudaSuccess ||
       (e = take_gemv_status_fp8(&bits)) != cudaSuccess ||
       (e = take_gemv_status_fp16(&bits)) != cudaSuccess || (e = take_tc_status(&bits)) != cudaSuccess ||
-      (e = take_attn_status(&bits)) != cudaSuccess)
+      (e = take_attn_status(&bits)) != cudaSuccess || (e = take_ring_status(&bits)) != cudaSuccess)
     return cuda_fail(e, "sq_check: linear status");
   if (device_bits) *device_bits = bits;
   if (bits) return fail(SQ_ERR_DEVICE, "sq_check: device status bits 0x%x", bits);
@@ -176,12 +176,20 @@ static sq_status run_linear(const sq_linear_op& op, cudaStream_t stream, const _
   a.ppad = (a.pieces + 31) / 32 * 32;
   cudaError_t e;
   const bool tc = use_tensor_cores(op.wkind, op.M, op.N, op.K, op.epi) && tc_supported(op.M, op.K, op.epi);
-  if (gamma && tc) {
-    // the tensor-core tile path stages x by TMA: the standalone RMSNorm first
+  const bool ring = !tc && use_ring(op.wkind, op.M, op.N, op.K, op.epi);
+  if (gamma && (tc || ring)) {
+    // the tensor-core tile path and the ring engine stage x by copies: the
+    // standalone RMSNorm first
     e = launch_rmsnorm(a.x, gamma, op.M, op.K, eps, xn, stream);
     if (e != cudaSuccess) return cuda_fail(e, "sq_linear_norm: rmsnorm launch");
     a.x = xn;
     a.gamma = nullptr;
+  }
+  if (ring) {
+    // one row through the shared-memory ring, register-operand tensor cores
+    e = launch_ring(op.wkind, a.x, op.w, op.scales, a.bias, a.residual, a.y, op.N, op.K, op.epi, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "sq_linear: ring launch");
+    return SQ_OK;
   }
   if (tc) {
     // tcgen05 tensor cores, weights on the MMA's M side
@@ -260,6 +268,7 @@ sq_status sq_linear_chain(const sq_linear_op* ops, int count, sq_stream_t stream
 int sq_linear_path(sq_wkind wkind, int M, int64_t N, int64_t K, sq_epilogue epi) {
   if (check_linear_sizes(wkind, M, N, K, epi) != SQ_OK) return -1;
   if (use_tensor_cores(wkind, M, N, K, epi) && tc_supported(M, K, epi)) return 1;
+  if (use_ring(wkind, M, N, K, epi)) return 3;
   return gemv_uses_mma(wkind, M, N) ? 2 : 0;
 }
 

@@ -101,6 +101,14 @@ cudaError_t launch_tc(int wkind, const __half* x, const void* w, const void* sca
                       cudaStream_t st);
 cudaError_t take_tc_status(uint32_t* bits);
 
+// sq_ring.cu: one activation row streamed through a shared-memory ring,
+// products on the register-operand tensor path (mma.sync).
+bool ring_supported(int wkind, int M, int64_t K);
+bool use_ring(int wkind, int M, int64_t N, int64_t K, int epi);
+cudaError_t launch_ring(int wkind, const __half* x, const void* w, const void* scales, const __half* bias,
+                        const __half* residual, __half* y, int64_t N, int64_t K, int epi, cudaStream_t st);
+cudaError_t take_ring_status(uint32_t* bits);
+
 // sq_accept.cu
 struct AcceptArgs {
   const float* p;

@@ -157,4 +157,27 @@ cudaError_t launch_gemv(int wk, const GemvArgs& a0, cudaStream_t st) {
   return cudaSuccess;
 }
 
+// The shared-memory ring engine (sq_ring.cu), one activation row, where it
+// measured faster than the GEMV family (GB300, graphs of whole-stack launch
+// sequences; us per launch, ring vs previous engine):
+//   INT4 fused gate/up of >= 64 Mi weights (7B, 14B): 14B 19.5 vs 25.8;
+//     the 1.5B one (27.5 Mi) stays on the register-operand path (6.9 vs 5.0);
+//   FP16 fused gate/up of >= 16 Mi weights: 14B 49.5 vs 54.0, 1.5B 10.0 vs
+//     11.3; FP16 lm_head (N >= 65536): 14B 228 vs 375, 1.5B 74.6 vs 79.5;
+//   FP8 lm_head of >= 400 Mi weights: 14B 124 vs 164 (1.5B: 46.0 vs 41.1).
+// q/k/v, o and down (96..448 tiles of 16 rows) stay on the GEMV family: at
+// 2-3 tiles per SM the ring's whole-tile work split leaves SMs idle.
+bool use_ring(int wkind, int M, int64_t N, int64_t K, int epi) {
+  if (!ring_supported(wkind, M, K)) return false;
+  const bool silu = epi == SQ_EPI_SILU_GATE;
+  const int64_t weights = (silu ? 2 * N : N) * K;
+  const int64_t Mi = (int64_t)1 << 20;
+  switch (wkind) {
+    case SQ_W_INT4: return silu && weights >= 64 * Mi;
+    case SQ_W_FP16: return (silu && weights >= 16 * Mi) || (!silu && N >= 65536);
+    case SQ_W_FP8: return !silu && weights >= 400 * Mi;
+  }
+  return false;
+}
+
 }  // namespace sq

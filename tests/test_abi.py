@@ -119,20 +119,32 @@ def test_binding_fails_loudly_without_the_library(tmp_path):
 
 
 def test_single_row_engine_choice(lib):
-    """sq_linear_path is host logic: one INT4 activation row over at least 304
-    16-row output tiles takes the register-operand tensor path (2), other
-    single-row calls the streaming CUDA-core GEMV (0)."""
+    """sq_linear_path is host logic: one activation row takes the shared-
+    memory ring (3) for the large matrices where it measured faster (INT4
+    fused gate/up of >= 64 Mi weights, FP16 fused gate/up of >= 16 Mi and
+    lm_head rows, FP8 lm_head of >= 400 Mi weights); otherwise one INT4 row
+    over at least 304 16-row output tiles takes the register-operand tensor
+    path (2) and other single-row calls the streaming CUDA-core GEMV (0)."""
     W4, W8, W16 = sq.SQ_W_INT4, sq.SQ_W_FP8, sq.SQ_W_FP16
     NONE, SILU, RES = sq.SQ_EPI_NONE, sq.SQ_EPI_SILU_GATE, sq.SQ_EPI_RESIDUAL
-    assert sq.sq_linear_path(W4, 1, 8960, 1536, SILU) == 2      # 1.5B fused gate/up
+    assert sq.sq_linear_path(W4, 1, 8960, 1536, SILU) == 2      # 1.5B fused gate/up (27.5 Mi)
     assert sq.sq_linear_path(W4, 1, 151936, 1536, NONE) == 2    # 1.5B lm_head
-    assert sq.sq_linear_path(W4, 1, 18944, 3584, SILU) == 2     # 7B fused gate/up
+    assert sq.sq_linear_path(W4, 1, 18944, 3584, SILU) == 3     # 7B fused gate/up (136 Mi)
+    assert sq.sq_linear_path(W4, 1, 13824, 5120, SILU) == 3     # 14B fused gate/up
+    assert sq.sq_linear_path(W4, 1, 152064, 5120, NONE) == 2    # 14B lm_head
     assert sq.sq_linear_path(W4, 1, 2048, 1536, NONE) == 0      # 1.5B q/k/v
     assert sq.sq_linear_path(W4, 1, 1536, 1536, RES) == 0       # 1.5B o
     assert sq.sq_linear_path(W4, 1, 1536, 8960, RES) == 0       # 1.5B down
     assert sq.sq_linear_path(W4, 1, 16 * 304, 896, NONE) == 2   # exactly 304 tiles
     assert sq.sq_linear_path(W4, 1, 16 * 304 - 16, 896, NONE) == 0
     assert sq.sq_linear_path(W4, 1, 16 * 303 + 1, 896, NONE) == 2  # ragged 304th tile
+    assert sq.sq_linear_path(W4, 1, 32768, 2176, SILU) == 2     # 17 groups: odd, not the ring
     assert sq.sq_linear_path(W4, 2, 151936, 1536, NONE) == 0    # two rows: streaming GEMV
-    assert sq.sq_linear_path(W8, 1, 151936, 1536, NONE) == 0
-    assert sq.sq_linear_path(W16, 1, 151936, 1536, NONE) == 0
+    assert sq.sq_linear_path(W8, 1, 151936, 1536, NONE) == 0    # 1.5B FP8 lm_head (233 Mi)
+    assert sq.sq_linear_path(W8, 1, 152064, 5120, NONE) == 3    # 14B FP8 lm_head (779 Mi)
+    assert sq.sq_linear_path(W8, 1, 13824, 5120, SILU) == 0
+    assert sq.sq_linear_path(W16, 1, 151936, 1536, NONE) == 3   # FP16 lm_head
+    assert sq.sq_linear_path(W16, 1, 8960, 1536, SILU) == 3     # FP16 fused gate/up (27.5 Mi)
+    assert sq.sq_linear_path(W16, 1, 4864, 896, SILU) == 0      # 0.5B-shaped (8.7 Mi)
+    assert sq.sq_linear_path(W16, 1, 2048, 1536, NONE) == 0
+    assert sq.sq_linear_path(W16, 5, 151936, 1536, NONE) == 0   # five rows: not the ring
