@@ -1,17 +1,25 @@
 #!/usr/bin/env python3
 """Benchmark of the SpecQuant draft/verify hot path on GB300.
 
-Workload (default): the Qwen2.5-1.5B-shaped linear stack (28 layers, hidden
-1536, 12 q / 2 kv heads, intermediate 8960, vocabulary 151936) with random
-fp16 weights ~ N(0, 0.02) and its INT4 and FP8 variants derived on the GPU;
-batch 1, K = 4 draft tokens.  One step is one speculative cycle:
+Workload (default): the Qwen2.5-14B-shaped linear stack (48 layers, hidden
+5120, 40 q / 8 kv heads, intermediate 13824, vocabulary 152064) with random
+fp16 weights ~ N(0, 0.02) and its INT4 and FP8 variants derived on the GPU,
+all three resident together; batch 1, K = 4 draft tokens.  One step is one
+speculative cycle:
   K draft passes of every projection + lm_head with the INT4 variant (M = 1),
+  each followed by sampling a draft token from its lm_head logits,
   one verify pass with the FP16 parent (M = K + 1 = 5),
-  one accept/resample over the vocabulary.
+  one accept/resample over the vocabulary from the passes' logits.
 The metric is tokens/s = B * E[tokens per cycle] / step time, with the mean
 number of tokens a cycle emits measured by sq_accept over a batch of
 synthetic speculative blocks (target logits ~ N(0, 2), draft logits =
 target + N(0, 0.5)).
+
+breakdown.per_config times the same cycle on every workload: the 0.5B-
+shaped MLP block (rotated copies, so that HBM and not L2 serves it), the
+1.5B stack, the 7B stack with INT4 drafts at K = 2, 4, 8 and with FP8
+drafts at batch 8 (48-row verify), and the 14B stack over batch 1, 4, 16
+and K = 4, 8.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -46,12 +54,14 @@ def parse():
     ap.add_argument("--steps", type=int, default=1000)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--workload", default="qwen2.5-1.5b")
+    ap.add_argument("--workload", default="qwen2.5-14b")
     ap.add_argument("--draft", choices=("int4", "fp8"), default="int4")
     ap.add_argument("--k", type=int, default=4, help="draft tokens per cycle")
     ap.add_argument("--batch", type=int, default=1, help="sequences per GPU")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="skip the per-workload breakdown (headline workload only)")
     ap.add_argument("--layers", type=int, default=None,
                     help="decoder layers to build (default: the workload's; --case runs only)")
     ap.add_argument("--case", default=None,
@@ -195,7 +205,8 @@ def kernel_digest(kernel_tag: str) -> str:
     engine, fmt = kernel_tag.split("_")[:2]
     files = {"gemv": ("sq_gemv.cuh", f"sq_gemv_{fmt}.cu"),
              "mma": ("sq_gemv.cuh", "sq_gemv_mma.cuh", f"sq_gemv_{fmt}.cu"),
-             "tc": ("sq_tc.cu",)}[engine] + _COMMON
+             "tc": ("sq_tc.cu",),
+             "ring": ("sq_ring.cu",)}[engine] + _COMMON
     return source_digest([os.path.join(_CSRC, f) for f in files])
 
 
@@ -211,6 +222,203 @@ def profiled_traffic(kernel_tag: str, digest: str):
         if m and t and m.group(1) == digest:
             return float(t.group(1))
     return None
+
+
+# ----------------------------------------------------------------------------- per-workload cycles
+
+_CAL = {}
+
+
+def mean_tokens_per_cycle(sq, torch, dev, K, V, draft_noise):
+    """E[tokens per cycle] of sq_accept over 64 synthetic blocks (target
+    logits N(0, 2); draft logits target + N(0, draft_noise), or independent
+    N(0, 2) when draft_noise is None), cached per (K, V, noise)."""
+    from paper_2609_21704_gb300 import synth
+
+    key = (K, V, draft_noise)
+    if key not in _CAL:
+        blk = [torch.from_numpy(a).to(dev) for a in synth.spec_block(99, 64, K, V, draft_noise=draft_noise)]
+        n = torch.empty(64, dtype=torch.int32, device=dev)
+        t = torch.empty(64, K + 1, dtype=torch.int32, device=dev)
+        ws = torch.zeros(sq.sq_accept_workspace_bytes(64, K, V), dtype=torch.uint8, device=dev)
+        sq.sq_accept(*blk, sq.SQ_ACCEPT_SAMPLE, n, t, ws)
+        if sq.sq_check() != 0:
+            raise RuntimeError("calibration accept flagged the device status word")
+        _CAL[key] = float(n.float().mean().item()) + 1.0
+    return _CAL[key]
+
+
+def measure_cycle(ctx, stack, draft, B, K, seed, reps, draft_noise=0.5):
+    """One speculative cycle on `stack`: K draft passes (M = B) each with a
+    draft sample from its logits, one FP16 verify pass (M = B (K + 1)), the
+    accept from the passes' logits; the whole cycle as one graph and each
+    piece alone.  Returns times (us), fractions of the HBM peak and
+    tokens/s = B * E[tokens per cycle] / cycle time."""
+    sq, stk, synth, torch = ctx["sq"], ctx["stk"], ctx["synth"], ctx["torch"]
+    dev, stream, capture, timed, peak = ctx["dev"], ctx["stream"], ctx["capture"], ctx["timed"], ctx["peak"]
+    V = stack.shape.vocab
+    Mv = B * (K + 1)
+    bd = stk.PassBuffers(stack, B, seed=seed + 1)
+    bv = stk.PassBuffers(stack, Mv, seed=seed + 2)
+    _, _, dr, u = synth.spec_block(seed + 3, B, K, V, draft_noise=draft_noise)
+    td, tu = torch.from_numpy(dr).to(dev), torch.from_numpy(u).to(dev)
+    zq = torch.empty(K, B, V, dtype=torch.float16, device=dev)
+    zp = bv.logits.view(B, K + 1, V)
+    u_draft = torch.from_numpy(synth.uniforms(seed + 4, (K, B))).to(dev)
+    samp = torch.empty(K, B, 1, dtype=torch.int32, device=dev)
+    n_out = torch.empty(B, dtype=torch.int32, device=dev)
+    tok_out = torch.empty(B, K + 1, dtype=torch.int32, device=dev)
+    ws_s = torch.zeros(sq.sq_accept_logits_workspace_bytes(B, 0, V), dtype=torch.uint8, device=dev)
+    ws_l = torch.zeros(sq.sq_accept_logits_workspace_bytes(B, K, V), dtype=torch.uint8, device=dev)
+
+    def step():
+        for k in range(K):
+            stk.run_pass(stack, draft, bd, stream, logits=zq[k])
+            sq.sq_sample_logits(zq[k], u_draft[k], 1.0, samp[k], ws_s, stream)
+        stk.run_pass(stack, "fp16", bv, stream)
+        sq.sq_accept_logits(zp, zq, td, tu, 1.0, sq.SQ_ACCEPT_SAMPLE, n_out, tok_out, ws_l, stream)
+
+    with torch.cuda.stream(stream):
+        g_step = capture(step)
+        g_d = capture(lambda: stk.run_pass(stack, draft, bd, stream, logits=zq[0]))
+        g_v = capture(lambda: stk.run_pass(stack, "fp16", bv, stream))
+        g_s = capture(lambda: sq.sq_sample_logits(zq[0], u_draft[0], 1.0, samp[0], ws_s, stream))
+        g_a = capture(lambda: sq.sq_accept_logits(zp, zq, td, tu, 1.0, sq.SQ_ACCEPT_SAMPLE, n_out, tok_out,
+                                                  ws_l, stream))
+        r_step = max(3, reps // max(1, K))
+        t_step = timed(g_step, r_step) / r_step
+        t_d = timed(g_d, reps) / reps
+        t_v = timed(g_v, reps) / reps
+        t_s = timed(g_s, reps) / reps
+        t_a = timed(g_a, reps) / reps
+    if sq.sq_check() != 0:
+        raise RuntimeError("a cycle flagged the device status word")
+    e_tok = mean_tokens_per_cycle(sq, torch, dev, K, V, draft_noise)
+    d_bytes = stack.weight_bytes(draft) + stack.activation_bytes(B)
+    v_bytes = stack.weight_bytes("fp16") + stack.activation_bytes(Mv)
+    del g_step, g_d, g_v, g_s, g_a, bd, bv
+    return {"B": B, "K": K, "draft": draft, "verify_rows": Mv,
+            "cycle_ms": 1e3 * t_step, "tokens_per_cycle": round(e_tok, 4),
+            "tokens_per_s": B * e_tok / t_step,
+            "draft_pass_us": 1e6 * t_d, "draft_pass_frac_of_peak": d_bytes / t_d / 1e9 / peak,
+            "verify_pass_us": 1e6 * t_v, "verify_pass_frac_of_peak": v_bytes / t_v / 1e9 / peak,
+            "sample_logits_us": 1e6 * t_s, "accept_logits_us": 1e6 * t_a}
+
+
+def measure_mlp_block(ctx, shape, K, reps, seed=0):
+    """The 0.5B-shaped MLP block (gate/up + SiLU, down): K INT4 draft steps at
+    M = 1, one FP16 verify at M = K + 1, sq_accept over V = 32000 on
+    synthetic probabilities with independent draft logits.  One block is
+    6.7 MB of INT4 and 26 MB of FP16, far inside the 129 MB L2, so the graphs
+    cycle through enough distinct copies of each (>= 4x L2 of each variant
+    between two uses of a copy) that every pass reads its weights from HBM."""
+    sq, synth, torch = ctx["sq"], ctx["synth"], ctx["torch"]
+    dev, stream, capture, timed, peak = ctx["dev"], ctx["stream"], ctx["capture"], ctx["timed"], ctx["peak"]
+    H, I, V = shape.hidden, shape.intermediate, 32000
+    l2x4 = 4 * 129 * 2 ** 20
+    cb, sb = sq.sq_quantized_bytes(sq.SQ_INT4_G128, 2 * I, H)
+    cb2, sb2 = sq.sq_quantized_bytes(sq.SQ_INT4_G128, H, I)
+    int4_bytes = cb + sb + cb2 + sb2
+    fp16_bytes = 2 * (2 * I * H + H * I)
+    n4, n16 = -(-l2x4 // int4_bytes), -(-l2x4 // fp16_bytes)
+    q4, w16s = [], []
+    for c in range(max(n4, n16)):
+        mats16, mats4 = [], []
+        for j, (n, k) in enumerate(((2 * I, H), (H, I))):
+            w16 = synth.weights_fp16_device(synth.stack_weight_seed(seed + 10 * c + j, 0), n, k, dev)
+            if c < n4:
+                codes = torch.empty(n, k // 2, dtype=torch.uint8, device=dev)
+                scales = torch.empty(n, k // 128, dtype=torch.float16, device=dev)
+                sq.sq_quantize(w16, sq.SQ_INT4_G128, codes, scales)
+                mats4.append((codes, scales))
+            mats16.append(w16)
+        if c < n4:
+            q4.append(mats4)
+        if c < n16:
+            w16s.append(mats16)
+        del mats16
+    Mv = K + 1
+    xd = synth.activations_fp16_device(seed + 1, 1, H, dev)
+    xv = synth.activations_fp16_device(seed + 2, Mv, H, dev)
+    hd = torch.empty(1, I, dtype=torch.float16, device=dev)
+    hv = torch.empty(Mv, I, dtype=torch.float16, device=dev)
+    yd = torch.empty(1, H, dtype=torch.float16, device=dev)
+    yv = torch.empty(Mv, H, dtype=torch.float16, device=dev)
+    p, q, dr, u = (torch.from_numpy(a).to(dev) for a in synth.spec_block(seed + 3, 1, K, V, draft_noise=None))
+    n_out = torch.empty(1, dtype=torch.int32, device=dev)
+    tok_out = torch.empty(1, K + 1, dtype=torch.int32, device=dev)
+    ws = torch.zeros(sq.sq_accept_workspace_bytes(1, K, V), dtype=torch.uint8, device=dev)
+
+    def draft_pass(c):
+        (gc, gs), (dc, ds) = q4[c % n4]
+        sq.sq_linear_chain([(sq.SQ_W_INT4, xd, gc, gs, None, None, sq.SQ_EPI_SILU_GATE, hd),
+                            (sq.SQ_W_INT4, hd, dc, ds, None, None, sq.SQ_EPI_NONE, yd)], stream)
+
+    def verify_pass(c):
+        gw, dw = w16s[c % n16]
+        sq.sq_linear_chain([(sq.SQ_W_FP16, xv, gw, None, None, None, sq.SQ_EPI_SILU_GATE, hv),
+                            (sq.SQ_W_FP16, hv, dw, None, None, None, sq.SQ_EPI_NONE, yv)], stream)
+
+    def accept():
+        sq.sq_accept(p, q, dr, u, sq.SQ_ACCEPT_SAMPLE, n_out, tok_out, ws, stream)
+
+    n_cycles = n16  # each cycle: K INT4 copies, one FP16 copy, in order
+
+    def cycles():
+        for i in range(n_cycles):
+            for k in range(K):
+                draft_pass(i * K + k)
+            verify_pass(i)
+            accept()
+    with torch.cuda.stream(stream):
+        g_c = capture(cycles)
+        g_d = capture(lambda: [draft_pass(c) for c in range(n4)])
+        g_v = capture(lambda: [verify_pass(c) for c in range(n16)])
+        g_a = capture(accept)
+        r = max(3, reps // 4)
+        t_c = timed(g_c, r) / (r * n_cycles)
+        t_d = timed(g_d, r) / (r * n4)
+        t_v = timed(g_v, r) / (r * n16)
+        t_a = timed(g_a, reps) / reps
+    if sq.sq_check() != 0:
+        raise RuntimeError("the MLP cycle flagged the device status word")
+    e_tok = mean_tokens_per_cycle(sq, torch, dev, K, V, None)
+    d_bytes = int4_bytes + 2 * (H + I + I + H)
+    v_bytes = fp16_bytes + 2 * Mv * (H + I + I + H)
+    del g_c, g_d, g_v, g_a, q4, w16s
+    return {"B": 1, "K": K, "draft": "int4", "verify_rows": Mv,
+            "copies_rotated": {"int4": n4, "fp16": n16},
+            "cycle_ms": 1e3 * t_c, "tokens_per_cycle": round(e_tok, 4), "tokens_per_s": e_tok / t_c,
+            "draft_pass_us": 1e6 * t_d, "draft_pass_frac_of_peak": d_bytes / t_d / 1e9 / peak,
+            "verify_pass_us": 1e6 * t_v, "verify_pass_frac_of_peak": v_bytes / t_v / 1e9 / peak,
+            "accept_us": 1e6 * t_a, "accept_vocab": V}
+
+
+def measure_all_configs(ctx, head_stack, reps):
+    """breakdown.per_config: every workload's cycle, driver-timed."""
+    stk, torch = ctx["stk"], ctx["torch"]
+    from paper_2609_21704_gb300.shapes import QWEN25_0P5B_MLP, QWEN25_1P5B, QWEN25_7B
+
+    out = {}
+    out["qwen2.5-0.5b-mlp int4 B=1 K=4"] = measure_mlp_block(ctx, QWEN25_0P5B_MLP, 4, reps)
+    st = stk.LinearStack(QWEN25_1P5B, ctx["dev"], seed=500, variants=("int4",))
+    out["qwen2.5-1.5b int4 B=1 K=4"] = measure_cycle(ctx, st, "int4", 1, 4, 510, reps)
+    del st
+    torch.cuda.empty_cache()
+    st = stk.LinearStack(QWEN25_7B, ctx["dev"], seed=700, variants=("int4", "fp8"))
+    for K in (2, 4, 8):
+        out[f"qwen2.5-7b int4 B=1 K={K}"] = measure_cycle(ctx, st, "int4", 1, K, 710 + K, reps)
+    out["qwen2.5-7b fp8 B=8 K=5"] = measure_cycle(ctx, st, "fp8", 8, 5, 720, reps)
+    del st
+    torch.cuda.empty_cache()
+    from paper_2609_21704_gb300.shapes import QWEN25_14B
+    st = head_stack if head_stack.shape.name == QWEN25_14B.name and len(head_stack.layers) == 48 else \
+        stk.LinearStack(QWEN25_14B, ctx["dev"], seed=1400, variants=("int4",))
+    for B in (1, 4, 16):
+        for K in (4, 8):
+            out[f"qwen2.5-14b int4 B={B} K={K}"] = measure_cycle(ctx, st, "int4", B, K, 900 + 10 * B + K,
+                                                                 max(5, reps // 4))
+    return out
 
 
 # ----------------------------------------------------------------------------- CPU oracle leg
@@ -608,6 +816,15 @@ def main():
             "speedup_vs_direct_fp16": (made_s / t_gs) / (made_d / t_gd),
             "distinct_tokens_per_sequence": distinct_s,
         }
+
+    # ---- every workload's cycle (N = 1 only: the scaling runs time the headline)
+    per_config = None
+    if world == 1 and not args.no_per_config:
+        mctx = {"sq": sq, "stk": stk, "synth": synth, "torch": torch, "dev": dev, "stream": stream,
+                "capture": capture, "timed": timed, "peak": peak_gbs}
+        t_pc = time.perf_counter()
+        per_config = measure_all_configs(mctx, stack, reps)
+        per_config["wall_s"] = round(time.perf_counter() - t_pc, 1)
     tensor_peak, tensor_peak_kind = measured_tensor_peak()
     pf_flops = 2.0 * 256 * stack.params()
     draft_bytes = stack.weight_bytes(args.draft) + stack.activation_bytes(B)
@@ -619,7 +836,7 @@ def main():
 
     # ---- dominant kernel: the fused gate/up + SiLU linear (largest per-launch
     # weight matrix in the layers); all layers' launches of it in one graph
-    engine = {1: "tc", 2: "mma"}.get(sq.sq_linear_path(stk.WKIND[args.draft], B, shape.intermediate,
+    engine = {1: "tc", 2: "mma", 3: "ring"}.get(sq.sq_linear_path(stk.WKIND[args.draft], B, shape.intermediate,
                                                       shape.hidden, sq.SQ_EPI_SILU_GATE), "gemv")
     kernel_tag = f"{engine}_{args.draft}_gateup_silu_m{B}"
     gu_projs = [layer[2] for layer in stack.layers]
@@ -744,6 +961,7 @@ def main():
             "decoder_direct_fp16_tokens_per_s": B * world / t_ddir,
             "decoder_speedup_vs_direct_fp16": (mean_tokens / t_dc) / (1.0 / t_ddir),
             "generation": gen,
+            "per_config": per_config,
             "prefill_m256_fp16_ms": 1e3 * t_pf16,
             "prefill_m256_fp16_tflops": pf_flops / t_pf16 / 1e12,
             "prefill_m256_%s_ms" % args.draft: 1e3 * t_pfd,
