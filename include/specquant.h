@@ -183,6 +183,20 @@ SQ_API sq_status sq_linear_norm(sq_wkind wkind, const void* x, const void* gamma
  * introspection for tests and tuning. */
 SQ_API int sq_linear_path(sq_wkind wkind, int M, int64_t N, int64_t K, sq_epilogue epi);
 
+/* Failure-path self-test (the paper has no counterpart).  Every wait inside
+ * the library's kernels is bounded; a wait that runs out sets SQ_DEV_TIMEOUT
+ * and the kernel finishes, so the device stays usable.  sq_selftest_wait
+ * makes one such wait run out on purpose: a one-thread kernel waits on an
+ * mbarrier that nothing ever arrives at, with nothing else in flight.
+ *   which = 0: the poll-bounded wait of the tcgen05 tile path, giving up
+ *              after `limit` polls (1 .. 2^24);
+ *   which = 1: the time-bounded wait of the shared-memory ring engine,
+ *              giving up after `limit` nanoseconds (1 .. 10^9).
+ * The next sq_check() reports SQ_ERR_DEVICE with SQ_DEV_TIMEOUT set (and
+ * clears it); the stream and the device stay usable.  Invalid arguments:
+ * SQ_ERR_INVALID_ARG, nothing launched. */
+SQ_API sq_status sq_selftest_wait(int which, uint64_t limit, sq_stream_t stream);
+
 /* Sec. III-D.2 / III-D.3: a draft or verify pass runs every projection of
  * every layer plus lm_head, one after another.  sq_linear_chain runs `count`
  * linear calls in order on `stream` with exactly the results of calling

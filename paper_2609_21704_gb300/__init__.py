@@ -27,6 +27,7 @@ __all__ = [
     "sq_quantized_bytes", "sq_quantize", "sq_linear_w4a16", "sq_linear_fp8", "sq_verify",
     "sq_linear_ex", "sq_accept_workspace_bytes", "sq_accept", "sq_sample", "sq_check",
     "sq_version", "sq_accept_noalloc", "sq_linear_path", "sq_linear_chain", "SqLinearOp",
+    "sq_selftest_wait",
     "sq_accept_logits_workspace_bytes", "sq_accept_logits", "sq_sample_logits",
     "sq_softmax_workspace_bytes", "sq_softmax", "sq_rmsnorm", "sq_kv_append",
     "sq_attention_workspace_bytes", "sq_attention", "sq_kv_rollback", "sq_embed",
@@ -65,6 +66,7 @@ _SIGS = {
     "sq_accept_noalloc": (_INT, [_P, _P, _P, _P, _INT, _INT, _I64, _INT, _P, _P, _P]),
     "sq_linear_path": (_INT, [_INT, _INT, _I64, _I64, _INT]),
     "sq_linear_chain": (_INT, [_P, _INT, _P]),
+    "sq_selftest_wait": (_INT, [_INT, ctypes.c_uint64, _P]),
     "sq_accept_logits_workspace_bytes": (_SIZE, [_INT, _INT, _I64]),
     "sq_accept_logits": (_INT, [_P, _P, _P, _P, _INT, _INT, _I64, ctypes.c_float, _INT, _P, _P, _P,
                                 _SIZE, _P]),
@@ -202,6 +204,12 @@ def _op_array(ops):
         arr[i] = SqLinearOp(wkind, epi, M, 0, y.shape[1], K, _ptr(x), _ptr(w), _ptr(scales),
                             _ptr(bias), _ptr(residual), _ptr(y))
     return arr
+
+
+def sq_selftest_wait(which: int, limit: int, stream=None) -> None:
+    """Make one bounded device wait run out (0: poll-bounded, `limit` polls;
+    1: time-bounded, `limit` ns); the next sq_check reports SQ_DEV_TIMEOUT."""
+    _check("sq_selftest_wait", load().sq_selftest_wait(which, limit, _stream(stream)))
 
 
 def sq_linear_w4a16(x, codes, scales, bias, y, stream=None) -> None:

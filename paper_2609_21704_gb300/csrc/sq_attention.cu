@@ -16,7 +16,7 @@
 // output rows [B*T, Hq D].  Token t of sequence b sits at position
 // pos0[b] + t.
 //
-// Attention is split over 64-key chunks of the cache (one CTA per
+// Attention is split over 32-key chunks of the cache (one CTA per
 // (sequence, key/value head, chunk)): all G * T queries of the group read
 // the chunk once from shared memory, then a combine kernel merges the
 // chunks' (max, sum, weighted value) partials.  Bound: the cache bytes

@@ -265,6 +265,18 @@ sq_status sq_linear_chain(const sq_linear_op* ops, int count, sq_stream_t stream
   return SQ_OK;
 }
 
+sq_status sq_selftest_wait(int which, uint64_t limit, sq_stream_t stream) {
+  if (which != 0 && which != 1) return fail(SQ_ERR_INVALID_ARG, "sq_selftest_wait: which must be 0 or 1");
+  if (which == 0 && (limit < 1 || limit > ((uint64_t)1 << 24)))
+    return fail(SQ_ERR_INVALID_ARG, "sq_selftest_wait: polls must be in [1, 2^24]");
+  if (which == 1 && (limit < 1 || limit > 1000000000ull))
+    return fail(SQ_ERR_INVALID_ARG, "sq_selftest_wait: limit must be in [1 ns, 1 s]");
+  cudaError_t e = which == 0 ? launch_wait_selftest_poll((uint32_t)limit, (cudaStream_t)stream)
+                             : launch_wait_selftest_time(limit, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "sq_selftest_wait: launch");
+  return SQ_OK;
+}
+
 int sq_linear_path(sq_wkind wkind, int M, int64_t N, int64_t K, sq_epilogue epi) {
   if (check_linear_sizes(wkind, M, N, K, epi) != SQ_OK) return -1;
   if (use_tensor_cores(wkind, M, N, K, epi) && tc_supported(M, K, epi)) return 1;
@@ -292,10 +304,12 @@ size_t sq_accept_workspace_bytes(int B, int K, int64_t V) {
   return accept_workspace_bytes(B, K, V);
 }
 
+// clear_counters: zero the ticket counters at the head of the workspace first
+// (the static scratch of sq_accept_noalloc), once every argument is valid.
 static sq_status accept_common(const char* who, const float* p, const float* q, const int32_t* draft,
                                const float* u, int B, int K, int64_t V, int mode, int32_t* n_accepted,
                                int32_t* tokens, void* workspace, size_t ws_bytes,
-                               sq_stream_t stream) {
+                               sq_stream_t stream, bool clear_counters = false) {
   if (mode != SQ_ACCEPT_SAMPLE && mode != SQ_ACCEPT_GREEDY)
     return fail(SQ_ERR_INVALID_ARG, "%s: unknown mode %d", who, mode);
   if (B < 0 || K < 0 || K > 16 || V < 1 || V >= ((int64_t)1 << 20))
@@ -330,7 +344,12 @@ static sq_status accept_common(const char* who, const float* p, const float* q, 
   a.C = (int)((V + kAcceptChunk - 1) / kAcceptChunk);
   a.chunk = kAcceptChunk;
   a.slots = K + 1 > 2 ? K + 1 : 2;
-  cudaError_t e = launch_accept(a, (cudaStream_t)stream);
+  cudaError_t e;
+  if (clear_counters) {
+    e = cudaMemsetAsync(workspace, 0, ctr, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "sq_accept: clearing the ticket counters");
+  }
+  e = launch_accept(a, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "sq_accept: launch");
   return SQ_OK;
 }
@@ -616,11 +635,10 @@ sq_status sq_accept_noalloc(const float* p, const float* q, const int32_t* draft
   void* scratch = nullptr;
   cudaError_t e = accept_noalloc_scratch(&scratch);
   if (e != cudaSuccess) return cuda_fail(e, "sq_accept_noalloc: scratch address");
-  const size_t ctr = (((size_t)B * 4u) + 15u) & ~(size_t)15u;
-  e = cudaMemsetAsync(scratch, 0, ctr, (cudaStream_t)stream);
-  if (e != cudaSuccess) return cuda_fail(e, "sq_accept_noalloc: clearing the ticket counters");
+  // the counters are cleared only after accept_common has accepted every
+  // argument: a rejected call queues nothing
   return accept_common("sq_accept_noalloc", p, q, draft, u, B, K, V, (int)mode, n_accepted, tokens,
-                       scratch, kAcceptNoallocScratchBytes, stream);
+                       scratch, kAcceptNoallocScratchBytes, stream, true);
 }
 
 }  // extern "C"

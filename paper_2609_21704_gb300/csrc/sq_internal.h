@@ -108,6 +108,9 @@ bool use_ring(int wkind, int M, int64_t N, int64_t K, int epi);
 cudaError_t launch_ring(int wkind, const __half* x, const void* w, const void* scales, const __half* bias,
                         const __half* residual, __half* y, int64_t N, int64_t K, int epi, cudaStream_t st);
 cudaError_t take_ring_status(uint32_t* bits);
+// Failure-path self-tests (sq_selftest_wait): a bounded wait that must run out.
+cudaError_t launch_wait_selftest_poll(uint32_t polls, cudaStream_t st);      // sq_tc.cu
+cudaError_t launch_wait_selftest_time(uint64_t limit_ns, cudaStream_t st);   // sq_ring.cu
 
 // sq_accept.cu
 struct AcceptArgs {

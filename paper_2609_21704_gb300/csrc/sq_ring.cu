@@ -569,6 +569,22 @@ cudaError_t launch_ring(int wkind, const __half* x, const void* w, const void* s
   }
 }
 
+// Failure-path self-test of the ring's timed wait: one thread waits on an
+// mbarrier that nothing arrives at, gives up after limit_ns nanoseconds and
+// sets SQ_DEV_TIMEOUT.  Nothing is in flight, so giving up is clean.
+__global__ void wait_selftest_time_kernel(uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  fence_mbar_init();
+  if (!mbar_wait_ns(&bar, 0, limit_ns)) atomicOr(&g_ring_status, SQ_DEV_TIMEOUT);
+}
+
+cudaError_t launch_wait_selftest_time(uint64_t limit_ns, cudaStream_t st) {
+  wait_selftest_time_kernel<<<1, 32, 0, st>>>(limit_ns);
+  return cudaGetLastError();
+}
+
 cudaError_t take_ring_status(uint32_t* bits) {
   unsigned int v = 0;
   cudaError_t e = cudaMemcpyFromSymbol(&v, g_ring_status, sizeof(v));

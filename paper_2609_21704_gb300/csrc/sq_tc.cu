@@ -758,6 +758,23 @@ cudaError_t launch_tc(int wk, const __half* x, const void* w, const void* scales
   return cudaErrorInvalidValue;
 }
 
+// Failure-path self-test: one thread waits, with the tile kernel's bounded
+// poll loop, on an mbarrier that nothing arrives at; after `polls` polls it
+// gives up and sets SQ_DEV_TIMEOUT, exactly as a tile kernel's wait would.
+// Nothing is in flight (no bulk copy, no MMA), so giving up is clean.
+__global__ void wait_selftest_poll_kernel(uint32_t polls) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  fence_mbar_init();
+  if (!mbar_wait_bounded(&bar, 0, polls)) atomicOr(&g_tc_status, SQ_DEV_TIMEOUT);
+}
+
+cudaError_t launch_wait_selftest_poll(uint32_t polls, cudaStream_t st) {
+  wait_selftest_poll_kernel<<<1, 32, 0, st>>>(polls);
+  return cudaGetLastError();
+}
+
 cudaError_t take_tc_status(uint32_t* bits) {
   uint32_t v = 0, zero = 0;
   cudaError_t e = cudaMemcpyFromSymbol(&v, g_tc_status, sizeof(v));

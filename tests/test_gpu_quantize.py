@@ -112,3 +112,16 @@ def test_nonfinite_weight_sets_status_bit():
     s8 = torch.empty(4, dtype=torch.float32, device=dev())
     sq.sq_quantize(wt, sq.SQ_FP8_E4M3_ROW, c8, s8)
     assert sq.sq_check() & sq.SQ_DEV_NONFINITE_WEIGHT
+
+
+def test_runs_on_sm_103a():
+    """The library carries sm_103a machine code only (no PTX to fall back
+    on), so a kernel that ran and gave bit-exact codes ran as sm_103a code
+    on a compute capability 10.3 device."""
+    assert torch.cuda.get_device_capability(dev()) == (10, 3)
+    w = synth.weights_fp16(3, 16, 128)
+    codes = torch.empty(16, 64, dtype=torch.uint8, device=dev())
+    scales = torch.empty(16, 1, dtype=torch.float16, device=dev())
+    sq.sq_quantize(f16_to_dev(w), sq.SQ_INT4_G128, codes, scales)
+    c, _ = oracle.quantize_int4(w.view(np.uint16))
+    assert np.array_equal(codes.cpu().numpy(), c)
