@@ -70,6 +70,7 @@ struct RingArgs {
   int32_t x_bytes;         // shared bytes of the staged activations
   int32_t K;
   int32_t ugran;           // parts of a row start on multiples of this many units
+  int32_t tmax;            // most tiles a CTA owns (ceil(T / grid))
 };
 
 static __device__ unsigned int g_ring_status;
@@ -119,31 +120,31 @@ __device__ __forceinline__ uint32_t slot_off(int r, int p, int rb) {
   return (uint32_t)(r * rb + ((p ^ ((r & 1) << 2)) << 4));
 }
 
-// A warp's position: round r (job tile), first unit u of the stage, end u1.
+// A warp's position: job j (tile ta + j / S, part j % S of its units), first
+// unit u of the stage, end unit u1 of the job.  Warp w takes the jobs w,
+// w + NW, w + 2 NW, ... of its CTA.
 struct Cur {
-  int r;
+  int j;
   int u, u1;
   int64_t tile;
   bool live;
 };
 
-template <int NW>
-__device__ __forceinline__ void cur_job(const RingArgs& a, int64_t ta, int64_t tb, int w, Cur& c) {
-  const int tpr = NW / a.S;
-  c.tile = ta + (int64_t)c.r * tpr + w / a.S;
+__device__ __forceinline__ void cur_job(const RingArgs& a, int64_t ta, int64_t tb, Cur& c) {
+  c.tile = ta + c.j / a.S;
   c.live = c.tile < tb;
-  const int p = w % a.S;
+  const int p = c.j % a.S;
   const int ug = a.ugran;  // INT4: parts start on even units (4-byte scale copies)
   c.u = ug * (p * (a.U / ug) / a.S);
   c.u1 = p + 1 == a.S ? a.U : ug * ((p + 1) * (a.U / ug) / a.S);
 }
 
 template <int NW, bool SILU>
-__device__ __forceinline__ void cur_next(const RingArgs& a, int64_t ta, int64_t tb, int w, Cur& c) {
+__device__ __forceinline__ void cur_next(const RingArgs& a, int64_t ta, int64_t tb, Cur& c) {
   c.u += SILU ? kUps32 : kUps16;
   if (c.u < c.u1) return;
-  ++c.r;
-  cur_job<NW>(a, ta, tb, w, c);
+  c.j += NW;
+  cur_job(a, ta, tb, c);
 }
 
 // Request the stage at c into slot `slot` with 16-byte asynchronous copies:
@@ -333,10 +334,15 @@ __global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const Rin
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int g = lane >> 2, t = lane & 3;
-  float* red = reinterpret_cast<float*>(smem + a.x_bytes);                             // [2][NW][32]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + a.x_bytes + 2 * NW * 32 * 4);   // [NW][ns]
+  // [x][partials: tmax * S * 32 fp32][arrival counters: tmax][mbarriers][slots][scale slots]
+  const int red_floats = a.S > 1 ? a.tmax * a.S * 32 : 0;
+  const int ncnt = a.S > 1 ? a.tmax : 0;
+  float* red = reinterpret_cast<float*>(smem + a.x_bytes);
+  int* cnt = reinterpret_cast<int*>(red + red_floats);
+  const int bar_off = a.x_bytes + red_floats * 4 + (ncnt * 4 + 15) / 16 * 16;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + bar_off);
   const uint32_t base = smem_u32(smem);
-  const uint32_t slot0 = (base + a.x_bytes + 2 * NW * 32 * 4 + NW * a.ns * 8 + 127) / 128 * 128;
+  const uint32_t slot0 = (base + bar_off + NW * a.ns * 8 + 127) / 128 * 128;
   uint64_t* mybar = bars + w * a.ns;
   const uint32_t xs_addr = base;
   const uint32_t slot_addr = slot0 + (uint32_t)(w * a.ns * kStageBytes);
@@ -345,29 +351,28 @@ __global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const Rin
 
   const int64_t ta = (int64_t)blockIdx.x * a.T / gridDim.x;
   const int64_t tb = (int64_t)(blockIdx.x + 1) * a.T / gridDim.x;
-  const int tpr = NW / a.S;
-  const int nr = (int)((tb - ta + tpr - 1) / tpr);
 
   if (lane == 0) {
     for (int i = 0; i < a.ns; ++i) mbar_init(&mybar[i], 32);  // one arrival per lane's copies
     fence_mbar_init();
   }
+  for (int i = threadIdx.x; i < ncnt; i += NW * 32) cnt[i] = 0;
   __syncwarp();
 
-  // ---- before the producer of x finishes: fill the ring, first scales
+  // ---- before the producer of x finishes: fill the ring
   Cur ic;
-  ic.r = 0;
-  cur_job<NW>(a, ta, tb, w, ic);
+  ic.j = w;
+  cur_job(a, ta, tb, ic);
   uint32_t issued = 0;
   for (int i = 0; i < a.ns && ic.live; ++i) {
     issue_stage<WK, SILU>(a, ic, slot_addr + (uint32_t)i * kStageBytes, sslot_addr + (uint32_t)i * kScaleBytes,
                           &mybar[i], lane);
-    cur_next<NW, SILU>(a, ta, tb, w, ic);
+    cur_next<NW, SILU>(a, ta, tb, ic);
     ++issued;
   }
   Cur cc;
-  cc.r = 0;
-  cur_job<NW>(a, ta, tb, w, cc);
+  cc.j = w;
+  cur_job(a, ta, tb, cc);
   // The next kernel is not signalled early: measured on the 14B INT4 draft
   // pass (8 layers), signalling at entry 660 us, before the epilogue 549 us,
   // at completion 483 us; FP16 / FP8 passes unchanged either way.
@@ -379,16 +384,16 @@ __global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const Rin
     uint4* xs = reinterpret_cast<uint4*>(smem);
     const int nch = a.K / 8;
     constexpr int B = 4;
-    for (int base = threadIdx.x; base < nch; base += NW * 32 * B) {
+    for (int b0 = threadIdx.x; b0 < nch; b0 += NW * 32 * B) {
       uint4 v[B];
 #pragma unroll
       for (int b = 0; b < B; ++b) {
-        const int c = base + b * NW * 32;
+        const int c = b0 + b * NW * 32;
         v[b] = c < nch ? reinterpret_cast<const uint4*>(a.x)[c] : make_uint4(0u, 0u, 0u, 0u);
       }
 #pragma unroll
       for (int b = 0; b < B; ++b) {
-        const int c = base + b * NW * 32;
+        const int c = b0 + b * NW * 32;
         if (c < nch) {
           if constexpr (WK == SQ_W_INT4)
             xs[(c >> 4) * 16 + (c & 3) * 4 + ((c >> 2) & 3)] = int4_x_order(v[b]);
@@ -402,20 +407,18 @@ __global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const Rin
 
   uint32_t status = 0, consumed = 0, broken_at = 0;
   bool broken = false;
-  for (int r = 0; r < nr; ++r) {
-    Cur job;
-    job.r = r;
-    cur_job<NW>(a, ta, tb, w, job);
+  while (cc.live) {
+    const Cur job = cc;
     float acc[2][2][4];
 #pragma unroll
     for (int h = 0; h < 2; ++h)
 #pragma unroll
       for (int c = 0; c < 2; ++c) acc[h][c][0] = acc[h][c][1] = acc[h][c][2] = acc[h][c][3] = 0.0f;
-    while (cc.live && cc.r == r) {
+    while (cc.live && cc.j == job.j) {
       const uint32_t k = consumed % (uint32_t)a.ns;
       const uint32_t parity = (consumed / (uint32_t)a.ns) & 1u;
       Cur nx = cc;
-      cur_next<NW, SILU>(a, ta, tb, w, nx);
+      cur_next<NW, SILU>(a, ta, tb, nx);
       const int nu = min(UPS, cc.u1 - cc.u);
       bool ok = false;
       if (!broken) {
@@ -443,19 +446,20 @@ __global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const Rin
       __syncwarp();
       if (!broken && ic.live) {
         issue_stage<WK, SILU>(a, ic, slot_addr + k * kStageBytes, sslot_addr + k * kScaleBytes, &mybar[k], lane);
-        cur_next<NW, SILU>(a, ta, tb, w, ic);
+        cur_next<NW, SILU>(a, ta, tb, ic);
         ++issued;
       }
       cc = nx;
     }
-    // rows g and g + 8 of the gate (h = 0) and up (h = 1) tiles
+    // ---- epilogue of the job: rows g and g + 8 of the gate (h = 0) and up
+    // (h = 1) tiles
     float v[2][2];
 #pragma unroll
     for (int h = 0; h < 2; ++h)
 #pragma unroll
       for (int rr = 0; rr < 2; ++rr) v[h][rr] = acc[h][0][2 * rr] + acc[h][1][2 * rr];
     if (a.S == 1) {
-      if (job.live && t == 0) {
+      if (t == 0) {
 #pragma unroll
         for (int rr = 0; rr < 2; ++rr) {
           const int64_t n = job.tile * 16 + pr + 8 * rr;
@@ -463,24 +467,34 @@ __global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const Rin
         }
       }
     } else {
-      float* rb = red + (r & 1) * NW * 32;
+      // the S parts of a tile meet in shared memory; the warp that completes
+      // the tile adds them in part order and stores
+      const int tl = (int)(job.tile - ta), part = job.j % a.S;
+      float* rp = red + (tl * a.S + part) * 32;
       if (t == 0) {
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
-          for (int rr = 0; rr < 2; ++rr) rb[w * 32 + h * 16 + g + 8 * rr] = v[h][rr];
+          for (int rr = 0; rr < 2; ++rr) rp[h * 16 + g + 8 * rr] = v[h][rr];
       }
-      __syncthreads();
-      if (job.live && w % a.S == 0 && t == 0) {
+      __threadfence_block();
+      __syncwarp();
+      int last = 0;
+      if (lane == 0) last = atomicAdd(&cnt[tl], 1) == a.S - 1;
+      last = __shfl_sync(0xffffffffu, last, 0);
+      if (last) {
+        __threadfence_block();
+        if (t == 0) {
 #pragma unroll
-        for (int rr = 0; rr < 2; ++rr) {
-          const int64_t n = job.tile * 16 + pr + 8 * rr;
-          float sv = 0.0f, su = 0.0f;
-          for (int s = 0; s < a.S; ++s) {
-            sv += rb[(w + s) * 32 + g + 8 * rr];
-            su += rb[(w + s) * 32 + 16 + g + 8 * rr];
+          for (int rr = 0; rr < 2; ++rr) {
+            const int64_t n = job.tile * 16 + pr + 8 * rr;
+            float sv = 0.0f, su = 0.0f;
+            for (int q = 0; q < a.S; ++q) {
+              sv += red[(tl * a.S + q) * 32 + g + 8 * rr];
+              su += red[(tl * a.S + q) * 32 + 16 + g + 8 * rr];
+            }
+            if (n < a.N) ring_store<WK, SILU>(a, n, sv, su);
           }
-          if (n < a.N) ring_store<WK, SILU>(a, n, sv, su);
         }
       }
     }
@@ -493,10 +507,11 @@ __global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const Rin
   if (status) atomicOr(&g_ring_status, status);
 }
 
-// Shared memory of one CTA of nw warps with ns slots per warp.
-size_t ring_smem(int nw, int x_bytes, int ns) {
+// Shared memory of one CTA of nw warps with ns slots per warp, x_bytes of
+// staged activations and red_floats fp32 partial sums with ncnt counters.
+size_t ring_smem(int nw, int x_bytes, int ns, int red_floats = 0, int ncnt = 0) {
   // + 128: the slots are aligned up to 128 bytes at run time
-  const int slot0 = x_bytes + 2 * nw * 32 * 4 + nw * ns * 8 + 128;
+  const int slot0 = x_bytes + red_floats * 4 + (ncnt * 4 + 15) / 16 * 16 + nw * ns * 8 + 128;
   return (size_t)slot0 + (size_t)nw * ns * (kStageBytes + kScaleBytes);
 }
 
@@ -527,7 +542,9 @@ bool ring_supported(int wkind, int M, int64_t K) {
   // INT4: an even number of groups per row (the scales travel in 4-byte copies)
   if (wkind == SQ_W_INT4 && (K / 128) % 2 != 0) return false;
   // at least two slots per warp beside the staged activations
-  return ring_smem(ring_warps(wkind), (int)((K * 2 + 127) / 128 * 128), 2) <= (size_t)ring_budget(wkind);
+  // (and up to 16 KB of partial sums with their counters)
+  return ring_smem(ring_warps(wkind), (int)((K * 2 + 127) / 128 * 128), 2, 4096, 128) <=
+         (size_t)ring_budget(wkind);
 }
 
 cudaError_t launch_ring(int wkind, const __half* x, const void* w, const void* scales, const __half* bias,
@@ -546,18 +563,43 @@ cudaError_t launch_ring(int wkind, const __half* x, const void* w, const void* s
   a.T = (N + 15) / 16;
   a.silu = epi == SQ_EPI_SILU_GATE;
   a.ugran = wkind == SQ_W_INT4 ? 2 : 1;
-  const int C = device_sm_count();
+  const int C0 = device_sm_count();
   const int nw = ring_warps(wkind);
-  int S = 1;
-  while (S < nw && 2 * S <= a.U / a.ugran && a.T * S < (int64_t)C * nw) S *= 2;
-  a.S = S;
+  const int grid = (int)(a.T < C0 ? a.T : C0);
+  a.tmax = (int32_t)((a.T + grid - 1) / grid);
+  // K split: each CTA owns whole tiles; its warps take (tile, part) jobs in
+  // turn.  FP16 / FP8 (memory-bound): S minimises the busiest warp's work,
+  // ceil(tmax S / nw) jobs of ceil(U / S) units plus about one unit of
+  // overhead per job (epilogue, partial sums).  INT4 (the SM's conversion
+  // throughput is the bound, not the busiest warp): the smallest S that gives
+  // three quarters of the warps a job (14B fused gate/up: S = 2; the
+  // balanced S = 8 measured 2.9 us slower per launch).  Within 16 KB of
+  // partial sums.
+  const int umax = a.U / a.ugran;
+  int best_s = 1;
+  int64_t best_cost = -1;
+  for (int S = 1; S <= umax && S <= 64; S *= 2) {
+    if (S > 1 && (int64_t)a.tmax * S * 32 * 4 > 16 * 1024) break;
+    if (wkind == SQ_W_INT4) {
+      best_s = S;
+      if ((int64_t)a.tmax * S * 4 >= 3 * nw) break;
+      continue;
+    }
+    const int64_t jobs = ((int64_t)a.tmax * S + nw - 1) / nw;
+    const int64_t cost = jobs * ((a.U + S - 1) / S + 1);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best_s = S;
+    }
+  }
+  a.S = best_s;
+  const int red_floats = a.S > 1 ? a.tmax * a.S * 32 : 0;
+  const int ncnt = a.S > 1 ? a.tmax : 0;
   a.x_bytes = (int32_t)((K * 2 + 127) / 128 * 128);
   int ns = 4;
-  while (ns > 2 && ring_smem(nw, a.x_bytes, ns) > (size_t)ring_budget(wkind)) --ns;
+  while (ns > 2 && ring_smem(nw, a.x_bytes, ns, red_floats, ncnt) > (size_t)ring_budget(wkind)) --ns;
   a.ns = ns;
-  const int64_t need = (a.T * S + nw - 1) / nw;  // CTAs that give every warp a job
-  const int grid = (int)(need < C ? need : C);
-  const size_t smem = ring_smem(nw, a.x_bytes, ns);
+  const size_t smem = ring_smem(nw, a.x_bytes, ns, red_floats, ncnt);
   const bool silu = a.silu != 0;
   switch (wkind) {
     case SQ_W_INT4:
