@@ -176,8 +176,9 @@ SQ_API sq_status sq_linear_norm(sq_wkind wkind, const void* x, const void* gamma
 /* Engine sq_linear_ex would use for these sizes: 1 = tcgen05 tensor cores,
  * 0 = CUDA-core GEMV, 2 = one INT4 activation row over at least 304 16-row
  * output tiles with the products on the tensor cores' register-operand path
- * (mma.sync), 3 = one activation row streamed through a shared-memory ring
- * of asynchronous copies, products on the same register-operand path,
+ * (mma.sync), 3 = one to eight activation rows streamed through a
+ * shared-memory ring of asynchronous copies, products on the same
+ * register-operand path,
  * -1 = sizes or kinds sq_linear_ex rejects (pointers are not examined;
  * nothing runs on the device).  The paper has no counterpart: this is
  * introspection for tests and tuning. */

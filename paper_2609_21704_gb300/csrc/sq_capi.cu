@@ -175,8 +175,11 @@ static sq_status run_linear(const sq_linear_op& op, cudaStream_t stream, const _
   a.pieces = (int)(op.K / weights_per_piece(op.wkind));
   a.ppad = (a.pieces + 31) / 32 * 32;
   cudaError_t e;
-  const bool tc = use_tensor_cores(op.wkind, op.M, op.N, op.K, op.epi) && tc_supported(op.M, op.K, op.epi);
-  const bool ring = !tc && use_ring(op.wkind, op.M, op.N, op.K, op.epi);
+  // the ring engine where the planner sends it, else the tcgen05 tile path,
+  // else the GEMV family (sq_plan.cu)
+  const bool ring = use_ring(op.wkind, op.M, op.N, op.K, op.epi);
+  const bool tc = !ring && use_tensor_cores(op.wkind, op.M, op.N, op.K, op.epi) &&
+                  tc_supported(op.M, op.K, op.epi);
   if (gamma && (tc || ring)) {
     // the tensor-core tile path and the ring engine stage x by copies: the
     // standalone RMSNorm first
@@ -186,8 +189,9 @@ static sq_status run_linear(const sq_linear_op& op, cudaStream_t stream, const _
     a.gamma = nullptr;
   }
   if (ring) {
-    // one row through the shared-memory ring, register-operand tensor cores
-    e = launch_ring(op.wkind, a.x, op.w, op.scales, a.bias, a.residual, a.y, op.N, op.K, op.epi, stream);
+    // one to eight rows through the shared-memory ring, register-operand tensor cores
+    e = launch_ring(op.wkind, a.x, op.w, op.scales, a.bias, a.residual, a.y, op.M, op.N, op.K, op.epi,
+                    stream);
     if (e != cudaSuccess) return cuda_fail(e, "sq_linear: ring launch");
     return SQ_OK;
   }
@@ -279,8 +283,8 @@ sq_status sq_selftest_wait(int which, uint64_t limit, sq_stream_t stream) {
 
 int sq_linear_path(sq_wkind wkind, int M, int64_t N, int64_t K, sq_epilogue epi) {
   if (check_linear_sizes(wkind, M, N, K, epi) != SQ_OK) return -1;
-  if (use_tensor_cores(wkind, M, N, K, epi) && tc_supported(M, K, epi)) return 1;
   if (use_ring(wkind, M, N, K, epi)) return 3;
+  if (use_tensor_cores(wkind, M, N, K, epi) && tc_supported(M, K, epi)) return 1;
   return gemv_uses_mma(wkind, M, N) ? 2 : 0;
 }
 

@@ -101,12 +101,13 @@ cudaError_t launch_tc(int wkind, const __half* x, const void* w, const void* sca
                       cudaStream_t st);
 cudaError_t take_tc_status(uint32_t* bits);
 
-// sq_ring.cu: one activation row streamed through a shared-memory ring,
-// products on the register-operand tensor path (mma.sync).
+// sq_ring.cu: one to eight activation rows streamed through a shared-memory
+// ring, products on the register-operand tensor path (mma.sync).
 bool ring_supported(int wkind, int M, int64_t K);
 bool use_ring(int wkind, int M, int64_t N, int64_t K, int epi);
 cudaError_t launch_ring(int wkind, const __half* x, const void* w, const void* scales, const __half* bias,
-                        const __half* residual, __half* y, int64_t N, int64_t K, int epi, cudaStream_t st);
+                        const __half* residual, __half* y, int M, int64_t N, int64_t K, int epi,
+                        cudaStream_t st);
 cudaError_t take_ring_status(uint32_t* bits);
 // Failure-path self-tests (sq_selftest_wait): a bounded wait that must run out.
 cudaError_t launch_wait_selftest_poll(uint32_t polls, cudaStream_t st);      // sq_tc.cu

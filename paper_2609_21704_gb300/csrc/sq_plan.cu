@@ -169,6 +169,12 @@ cudaError_t launch_gemv(int wk, const GemvArgs& a0, cudaStream_t st) {
 // 2-3 tiles per SM the ring's whole-tile work split leaves SMs idle.
 bool use_ring(int wkind, int M, int64_t N, int64_t K, int epi) {
   if (!ring_supported(wkind, M, K)) return false;
+  // two to eight rows cost the products of one on the ring: INT4 and FP8
+  // take it there, ahead of the tcgen05 tiles too (14B 8-layer passes, us:
+  // INT4 at 4 rows 1197 -> 655, at 8 rows 1099 -> 880; FP8 at 4 rows
+  // 1067 -> 872, at 8 rows 1271 -> 946); FP16 stays on the GEMV and the
+  // tiles (ring 1228 -> 1264 at 4 rows, 1229 -> 1283 at 8)
+  if (M > 1) return wkind != SQ_W_FP16;
   const bool silu = epi == SQ_EPI_SILU_GATE;
   const int64_t weights = (silu ? 2 * N : N) * K;
   const int64_t Mi = (int64_t)1 << 20;

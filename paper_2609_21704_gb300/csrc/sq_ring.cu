@@ -1,6 +1,7 @@
-// sq_ring.cu -- linear layer for ONE activation row (the draft pass at batch
-// 1, Sec. III-D.2) streamed through a shared-memory ring, products on the
-// tensor cores' register-operand path.
+// sq_ring.cu -- linear layer for one to eight activation rows (the draft
+// pass at small batch, Sec. III-D.2; the verify pass of one sequence, Sec.
+// III-D.3) streamed through a shared-memory ring, products on the tensor
+// cores' register-operand path.
 //
 // Used for the large single-row matrices (fused gate/up, lm_head) where it
 // measured faster than the GEMV family; the engine rule is in sq_plan.cu.
@@ -18,8 +19,9 @@
 //     x (weights never depend on it);
 //   * products: mma.sync m16n8k16, fp16 x fp16 -> fp32.  A = 16 weight rows
 //     from the slot (INT4 nibbles and E4M3 codes turned into exact fp16
-//     values in registers), B = the activation row, the same in all eight
-//     columns, so any column of D holds the 16 dot products.  INT4 groups
+//     values in registers), B = up to eight activation rows, one per column
+//     (lanes of columns past M read row M - 1; those columns are dropped),
+//     so M <= 8 rows cost the instructions of one.  INT4 groups
 //     are summed from zero in four (fused gate/up: two) independent
 //     accumulators and scaled by the group's fp16 scale into an fp32 sum;
 //     the scales travel with the stage (4-byte copies into a 128-byte scale
@@ -38,9 +40,9 @@ namespace sq {
 
 namespace {
 
-// Warps per CTA: 8 for FP16 / FP8 (memory-bound; at most half an SM's
-// shared memory), 16 for INT4 (bound by the nibble conversion: the whole
-// SM's warps hide its latency; 8 warps measured 1.3x slower).
+// Warps per CTA: 8 for FP16 / FP8 (memory-bound), 16 for INT4 (bound by the
+// nibble conversion: the whole SM's warps hide its latency; 8 warps measured
+// 1.3x slower) unless the staged activations leave no room for them.
 constexpr int kWarpsHalf = 8;
 constexpr int kWarpsFull = 16;
 constexpr int kStageBytes = 4096;          // weights of one ring slot
@@ -48,18 +50,17 @@ constexpr int kScaleBytes = 128;           // INT4 group scales of one slot
 constexpr int kUnitBytes = 64;             // a unit: 64 bytes of one weight row
 constexpr int kUps16 = 4;                  // units per stage of 16 rows
 constexpr int kUps32 = 2;                  // units per stage of 32 rows (fused gate/up)
-constexpr int kSmemHalf = 110 * 1024;      // under half an SM
 constexpr int kSmemFull = 227 * 1024;     // the whole opt-in shared memory of an SM
 constexpr uint64_t kWaitNs = 2000000000ull;
 constexpr uint64_t kDrainNs = 1000000ull;
 
 struct RingArgs {
-  const __half* x;         // [1, K]
+  const __half* x;         // [M, K]
   const uint8_t* w;        // weight rows
   const void* scales;      // INT4 fp16 [rows, K/128]; FP8 fp32 [rows]; FP16 unused
   const __half* bias;      // [rows] or null
-  const __half* residual;  // [1, N] or null
-  __half* y;               // [1, N]
+  const __half* residual;  // [M, N] or null
+  __half* y;               // [M, N]
   int64_t N;               // output columns
   int64_t row_bytes;
   int64_t T;               // 16-column output tiles
@@ -71,6 +72,8 @@ struct RingArgs {
   int32_t K;
   int32_t ugran;           // parts of a row start on multiples of this many units
   int32_t tmax;            // most tiles a CTA owns (ceil(T / grid))
+  int32_t M;               // activation rows, 1 .. 8 (the MMA's N columns)
+  int32_t x_stride;        // shared bytes between staged activation rows
 };
 
 static __device__ unsigned int g_ring_status;
@@ -255,13 +258,12 @@ __device__ __forceinline__ void stage_int4(uint32_t slot, uint32_t sslot, int nu
         // (row pr, row pr + 8) scales of unit u
         const uint32_t spair = __byte_perm(sw[h][0][u >> 1], sw[h][1][u >> 1], (u & 1) ? 0x7632 : 0x5410);
         const float2 s = __half22float2(*reinterpret_cast<const __half2*>(&spair));
-        float r0 = d[h][0][0] + d[h][1][0], r8 = d[h][0][2] + d[h][1][2];
-        if constexpr (NC == 4) {
-          r0 += d[h][2][0] + d[h][3][0];
-          r8 += d[h][2][2] + d[h][3][2];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {  // (row pr | pr + 8) x (column 2t | 2t + 1)
+          float r = d[h][0][e] + d[h][1][e];
+          if constexpr (NC == 4) r += d[h][2][e] + d[h][3][e];
+          acc[h][0][e] = fmaf(e < 2 ? s.x : s.y, r, acc[h][0][e]);
         }
-        acc[h][0][0] = fmaf(s.x, r0, acc[h][0][0]);
-        acc[h][0][2] = fmaf(s.y, r8, acc[h][0][2]);
       }
     }
   }
@@ -316,7 +318,7 @@ __device__ __forceinline__ void stage_fp8(uint32_t slot, int nu, int ug, uint32_
 // y[n] from the fp32 dot product v (and the up row's u): FP8 row scale,
 // bias, silu(v) * u, residual, fp16 -- the order of the GEMV kernels.
 template <int WK, bool SILU>
-__device__ __forceinline__ void ring_store(const RingArgs& a, int64_t n, float v, float u) {
+__device__ __forceinline__ void ring_store(const RingArgs& a, int64_t n, int m, float v, float u) {
   if constexpr (WK == SQ_W_FP8) v *= reinterpret_cast<const float*>(a.scales)[n];
   if (a.bias) v += __half2float(a.bias[n]);
   if constexpr (SILU) {
@@ -324,8 +326,8 @@ __device__ __forceinline__ void ring_store(const RingArgs& a, int64_t n, float v
     if (a.bias) u += __half2float(a.bias[a.N + n]);
     v = v / (1.0f + expf(-v)) * u;
   }
-  if (a.residual) v += __half2float(a.residual[n]);
-  a.y[n] = __float2half_rn(v);
+  if (a.residual) v += __half2float(a.residual[(int64_t)m * a.N + n]);
+  a.y[(int64_t)m * a.N + n] = __float2half_rn(v);
 }
 
 template <int WK, bool SILU, int NW>
@@ -335,7 +337,8 @@ __global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const Rin
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int g = lane >> 2, t = lane & 3;
   // [x][partials: tmax * S * 32 fp32][arrival counters: tmax][mbarriers][slots][scale slots]
-  const int red_floats = a.S > 1 ? a.tmax * a.S * 32 : 0;
+  const int pb = 32 * a.M;  // floats of one job's partial sums: [tile h][row][column]
+  const int red_floats = a.S > 1 ? a.tmax * a.S * pb : 0;
   const int ncnt = a.S > 1 ? a.tmax : 0;
   float* red = reinterpret_cast<float*>(smem + a.x_bytes);
   int* cnt = reinterpret_cast<int*>(red + red_floats);
@@ -344,7 +347,8 @@ __global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const Rin
   const uint32_t base = smem_u32(smem);
   const uint32_t slot0 = (base + bar_off + NW * a.ns * 8 + 127) / 128 * 128;
   uint64_t* mybar = bars + w * a.ns;
-  const uint32_t xs_addr = base;
+  // this lane's activation row: column g of B (columns past M repeat row M - 1)
+  const uint32_t xs_addr = base + (uint32_t)((g < a.M ? g : a.M - 1) * a.x_stride);
   const uint32_t slot_addr = slot0 + (uint32_t)(w * a.ns * kStageBytes);
   const uint32_t sslot_addr = slot0 + (uint32_t)(NW * a.ns * kStageBytes + w * a.ns * kScaleBytes);
   const int pr = g;  // rows g and g + 8 of the tile
@@ -381,20 +385,22 @@ __global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const Rin
   // ---- stage x: INT4 in the conversion's pair order with unit j's chunk
   // (t, q) at slot j * 16 + q * 4 + t; FP8 and FP16 in natural order
   {
-    uint4* xs = reinterpret_cast<uint4*>(smem);
-    const int nch = a.K / 8;
+    const int nch = a.K / 8;  // 16-byte chunks of one row
+    const int total = a.M * nch;
     constexpr int B = 4;
-    for (int b0 = threadIdx.x; b0 < nch; b0 += NW * 32 * B) {
+    for (int b0 = threadIdx.x; b0 < total; b0 += NW * 32 * B) {
       uint4 v[B];
 #pragma unroll
       for (int b = 0; b < B; ++b) {
-        const int c = b0 + b * NW * 32;
-        v[b] = c < nch ? reinterpret_cast<const uint4*>(a.x)[c] : make_uint4(0u, 0u, 0u, 0u);
+        const int i = b0 + b * NW * 32;
+        v[b] = i < total ? reinterpret_cast<const uint4*>(a.x)[i] : make_uint4(0u, 0u, 0u, 0u);
       }
 #pragma unroll
       for (int b = 0; b < B; ++b) {
-        const int c = b0 + b * NW * 32;
-        if (c < nch) {
+        const int i = b0 + b * NW * 32;
+        if (i < total) {
+          const int m = i / nch, c = i - m * nch;
+          uint4* xs = reinterpret_cast<uint4*>(smem + m * a.x_stride);
           if constexpr (WK == SQ_W_INT4)
             xs[(c >> 4) * 16 + (c & 3) * 4 + ((c >> 2) & 3)] = int4_x_order(v[b]);
           else
@@ -451,31 +457,33 @@ __global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const Rin
       }
       cc = nx;
     }
-    // ---- epilogue of the job: rows g and g + 8 of the gate (h = 0) and up
-    // (h = 1) tiles
-    float v[2][2];
+    // ---- epilogue of the job: D register e of tile h (gate / up) is row
+    // pr + 8 (e >> 1), activation row (column) 2t + (e & 1)
+    float v[2][4];
 #pragma unroll
     for (int h = 0; h < 2; ++h)
 #pragma unroll
-      for (int rr = 0; rr < 2; ++rr) v[h][rr] = acc[h][0][2 * rr] + acc[h][1][2 * rr];
+      for (int e = 0; e < 4; ++e) v[h][e] = acc[h][0][e] + acc[h][1][e];
     if (a.S == 1) {
-      if (t == 0) {
 #pragma unroll
-        for (int rr = 0; rr < 2; ++rr) {
-          const int64_t n = job.tile * 16 + pr + 8 * rr;
-          if (n < a.N) ring_store<WK, SILU>(a, n, v[0][rr], v[1][rr]);
-        }
+      for (int e = 0; e < 4; ++e) {
+        const int m = 2 * t + (e & 1);
+        const int64_t n = job.tile * 16 + pr + 8 * (e >> 1);
+        if (m < a.M && n < a.N) ring_store<WK, SILU>(a, n, m, v[0][e], v[1][e]);
       }
     } else {
       // the S parts of a tile meet in shared memory; the warp that completes
       // the tile adds them in part order and stores
       const int tl = (int)(job.tile - ta), part = job.j % a.S;
-      float* rp = red + (tl * a.S + part) * 32;
-      if (t == 0) {
+      float* rp = red + (tl * a.S + part) * pb;
 #pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-          for (int rr = 0; rr < 2; ++rr) rp[h * 16 + g + 8 * rr] = v[h][rr];
+      for (int e = 0; e < 4; ++e) {
+        const int m = 2 * t + (e & 1);
+        const int row = pr + 8 * (e >> 1);
+        if (m < a.M) {
+          rp[row * a.M + m] = v[0][e];
+          rp[(16 + row) * a.M + m] = v[1][e];
+        }
       }
       __threadfence_block();
       __syncwarp();
@@ -484,16 +492,18 @@ __global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const Rin
       last = __shfl_sync(0xffffffffu, last, 0);
       if (last) {
         __threadfence_block();
-        if (t == 0) {
 #pragma unroll
-          for (int rr = 0; rr < 2; ++rr) {
-            const int64_t n = job.tile * 16 + pr + 8 * rr;
+        for (int e = 0; e < 4; ++e) {
+          const int m = 2 * t + (e & 1);
+          const int row = pr + 8 * (e >> 1);
+          const int64_t n = job.tile * 16 + row;
+          if (m < a.M && n < a.N) {
             float sv = 0.0f, su = 0.0f;
             for (int q = 0; q < a.S; ++q) {
-              sv += red[(tl * a.S + q) * 32 + g + 8 * rr];
-              su += red[(tl * a.S + q) * 32 + 16 + g + 8 * rr];
+              sv += red[(tl * a.S + q) * pb + row * a.M + m];
+              su += red[(tl * a.S + q) * pb + (16 + row) * a.M + m];
             }
-            if (n < a.N) ring_store<WK, SILU>(a, n, sv, su);
+            ring_store<WK, SILU>(a, n, m, sv, su);
           }
         }
       }
@@ -515,12 +525,25 @@ size_t ring_smem(int nw, int x_bytes, int ns, int red_floats = 0, int ncnt = 0) 
   return (size_t)slot0 + (size_t)nw * ns * (kStageBytes + kScaleBytes);
 }
 
-int ring_warps(int wkind) { return wkind == SQ_W_INT4 ? kWarpsFull : kWarpsHalf; }
-int ring_budget(int wkind) { return wkind == SQ_W_INT4 ? kSmemFull : kSmemHalf; }
+// Staged activation rows: K fp16 each, rows 64 bytes past a multiple of 128
+// apart when there are several (lanes of columns 2i and 2i + 1 then read
+// different bank halves).
+int ring_x_stride(int M, int64_t K) {
+  const int row = (int)((K * 2 + 127) / 128 * 128);
+  return M > 1 ? row + 64 : row;
+}
+int ring_x_bytes(int M, int64_t K) { return (M * ring_x_stride(M, K) + 127) / 128 * 128; }
 
-template <int WK, bool SILU>
+// Warps per CTA: 8 for FP16 / FP8; 16 for INT4 when two slots per warp fit
+// beside the staged activations, else 8.
+int ring_warps(int wkind, int M, int64_t K) {
+  if (wkind != SQ_W_INT4) return kWarpsHalf;
+  return ring_smem(kWarpsFull, ring_x_bytes(M, K), 2, 4096, 128) <= (size_t)kSmemFull ? kWarpsFull
+                                                                                      : kWarpsHalf;
+}
+
+template <int WK, bool SILU, int NW>
 cudaError_t launch_inst(const RingArgs& a, size_t smem, int grid, cudaStream_t st) {
-  constexpr int NW = WK == SQ_W_INT4 ? kWarpsFull : kWarpsHalf;
   auto k = ring_linear_kernel<WK, SILU, NW>;
   static bool attr_set[64] = {false};
   int dev = 0;
@@ -528,27 +551,39 @@ cudaError_t launch_inst(const RingArgs& a, size_t smem, int grid, cudaStream_t s
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (!attr_set[dev]) {
-    e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, ring_budget(WK));
+    e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemFull);
     if (e != cudaSuccess) return e;
     attr_set[dev] = true;
   }
   return launch_pdl(k, dim3(grid), dim3(NW * 32), smem, st, a);
 }
 
+template <int WK>
+cudaError_t launch_wk(const RingArgs& a, int nw, size_t smem, int grid, cudaStream_t st) {
+  const bool silu = a.silu != 0;
+  if constexpr (WK == SQ_W_INT4) {
+    if (nw == kWarpsFull)
+      return silu ? launch_inst<WK, true, kWarpsFull>(a, smem, grid, st)
+                  : launch_inst<WK, false, kWarpsFull>(a, smem, grid, st);
+  }
+  return silu ? launch_inst<WK, true, kWarpsHalf>(a, smem, grid, st)
+              : launch_inst<WK, false, kWarpsHalf>(a, smem, grid, st);
+}
+
 }  // namespace
 
 bool ring_supported(int wkind, int M, int64_t K) {
-  if (M != 1 || K % 128 != 0) return false;
+  if (M < 1 || M > 8 || K % 128 != 0) return false;
   // INT4: an even number of groups per row (the scales travel in 4-byte copies)
   if (wkind == SQ_W_INT4 && (K / 128) % 2 != 0) return false;
-  // at least two slots per warp beside the staged activations
-  // (and up to 16 KB of partial sums with their counters)
-  return ring_smem(ring_warps(wkind), (int)((K * 2 + 127) / 128 * 128), 2, 4096, 128) <=
-         (size_t)ring_budget(wkind);
+  // at least two slots per warp beside the staged activations (and up to 16 KB
+  // of partial sums with their counters)
+  return ring_smem(ring_warps(wkind, M, K), ring_x_bytes(M, K), 2, 4096, 128) <= (size_t)kSmemFull;
 }
 
 cudaError_t launch_ring(int wkind, const __half* x, const void* w, const void* scales, const __half* bias,
-                        const __half* residual, __half* y, int64_t N, int64_t K, int epi, cudaStream_t st) {
+                        const __half* residual, __half* y, int M, int64_t N, int64_t K, int epi,
+                        cudaStream_t st) {
   RingArgs a = {};
   a.x = x;
   a.w = reinterpret_cast<const uint8_t*>(w);
@@ -556,6 +591,7 @@ cudaError_t launch_ring(int wkind, const __half* x, const void* w, const void* s
   a.bias = bias;
   a.residual = residual;
   a.y = y;
+  a.M = M;
   a.N = N;
   a.K = (int32_t)K;
   a.row_bytes = row_bytes_of(wkind, K);
@@ -564,7 +600,7 @@ cudaError_t launch_ring(int wkind, const __half* x, const void* w, const void* s
   a.silu = epi == SQ_EPI_SILU_GATE;
   a.ugran = wkind == SQ_W_INT4 ? 2 : 1;
   const int C0 = device_sm_count();
-  const int nw = ring_warps(wkind);
+  const int nw = ring_warps(wkind, M, K);
   const int grid = (int)(a.T < C0 ? a.T : C0);
   a.tmax = (int32_t)((a.T + grid - 1) / grid);
   // K split: each CTA owns whole tiles; its warps take (tile, part) jobs in
@@ -579,7 +615,7 @@ cudaError_t launch_ring(int wkind, const __half* x, const void* w, const void* s
   int best_s = 1;
   int64_t best_cost = -1;
   for (int S = 1; S <= umax && S <= 64; S *= 2) {
-    if (S > 1 && (int64_t)a.tmax * S * 32 * 4 > 16 * 1024) break;
+    if (S > 1 && (int64_t)a.tmax * S * 32 * M * 4 > 16 * 1024) break;
     if (wkind == SQ_W_INT4) {
       best_s = S;
       if ((int64_t)a.tmax * S * 4 >= 3 * nw) break;
@@ -593,21 +629,18 @@ cudaError_t launch_ring(int wkind, const __half* x, const void* w, const void* s
     }
   }
   a.S = best_s;
-  const int red_floats = a.S > 1 ? a.tmax * a.S * 32 : 0;
+  const int red_floats = a.S > 1 ? a.tmax * a.S * 32 * M : 0;
   const int ncnt = a.S > 1 ? a.tmax : 0;
-  a.x_bytes = (int32_t)((K * 2 + 127) / 128 * 128);
+  a.x_stride = ring_x_stride(M, K);
+  a.x_bytes = ring_x_bytes(M, K);
   int ns = 4;
-  while (ns > 2 && ring_smem(nw, a.x_bytes, ns, red_floats, ncnt) > (size_t)ring_budget(wkind)) --ns;
+  while (ns > 2 && ring_smem(nw, a.x_bytes, ns, red_floats, ncnt) > (size_t)kSmemFull) --ns;
   a.ns = ns;
   const size_t smem = ring_smem(nw, a.x_bytes, ns, red_floats, ncnt);
-  const bool silu = a.silu != 0;
   switch (wkind) {
-    case SQ_W_INT4:
-      return silu ? launch_inst<SQ_W_INT4, true>(a, smem, grid, st) : launch_inst<SQ_W_INT4, false>(a, smem, grid, st);
-    case SQ_W_FP8:
-      return silu ? launch_inst<SQ_W_FP8, true>(a, smem, grid, st) : launch_inst<SQ_W_FP8, false>(a, smem, grid, st);
-    default:
-      return silu ? launch_inst<SQ_W_FP16, true>(a, smem, grid, st) : launch_inst<SQ_W_FP16, false>(a, smem, grid, st);
+    case SQ_W_INT4: return launch_wk<SQ_W_INT4>(a, nw, smem, grid, st);
+    case SQ_W_FP8: return launch_wk<SQ_W_FP8>(a, nw, smem, grid, st);
+    default: return launch_wk<SQ_W_FP16>(a, nw, smem, grid, st);
   }
 }
 

@@ -127,9 +127,12 @@ def test_single_row_engine_choice(lib):
     """sq_linear_path is host logic: one activation row takes the shared-
     memory ring (3) for the large matrices where it measured faster (INT4
     fused gate/up of >= 64 Mi weights, FP16 fused gate/up of >= 16 Mi and
-    lm_head rows, FP8 lm_head of >= 400 Mi weights); otherwise one INT4 row
+    lm_head rows, FP8 lm_head of >= 400 Mi weights), two to eight INT4 or
+    FP8 rows take it whenever their activations fit; otherwise one INT4 row
     over at least 304 16-row output tiles takes the register-operand tensor
-    path (2) and other single-row calls the streaming CUDA-core GEMV (0)."""
+    path (2) and other few-row calls the streaming CUDA-core GEMV (0).  (The
+    tcgen05 path (1) needs a device to encode its tensor maps: checked in
+    tests/test_gpu_tc.py.)"""
     W4, W8, W16 = sq.SQ_W_INT4, sq.SQ_W_FP8, sq.SQ_W_FP16
     NONE, SILU, RES = sq.SQ_EPI_NONE, sq.SQ_EPI_SILU_GATE, sq.SQ_EPI_RESIDUAL
     assert sq.sq_linear_path(W4, 1, 8960, 1536, SILU) == 2      # 1.5B fused gate/up (27.5 Mi)
@@ -144,7 +147,10 @@ def test_single_row_engine_choice(lib):
     assert sq.sq_linear_path(W4, 1, 16 * 304 - 16, 896, NONE) == 0
     assert sq.sq_linear_path(W4, 1, 16 * 303 + 1, 896, NONE) == 2  # ragged 304th tile
     assert sq.sq_linear_path(W4, 1, 32768, 2176, SILU) == 2     # 17 groups: odd, not the ring
-    assert sq.sq_linear_path(W4, 2, 151936, 1536, NONE) == 0    # two rows: streaming GEMV
+    assert sq.sq_linear_path(W4, 2, 151936, 1536, NONE) == 3    # two rows: the ring too
+    assert sq.sq_linear_path(W8, 8, 7168, 5120, NONE) == 3      # FP8 draft at batch 8
+    assert sq.sq_linear_path(W16, 2, 2048, 1536, NONE) == 0     # FP16 rows: not the ring
+    assert sq.sq_linear_path(W4, 9, 2048, 1536, NONE) == 0      # nine rows: not the ring
     assert sq.sq_linear_path(W8, 1, 151936, 1536, NONE) == 0    # 1.5B FP8 lm_head (233 Mi)
     assert sq.sq_linear_path(W8, 1, 152064, 5120, NONE) == 3    # 14B FP8 lm_head (779 Mi)
     assert sq.sq_linear_path(W8, 1, 13824, 5120, SILU) == 0

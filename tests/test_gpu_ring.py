@@ -2,7 +2,8 @@
 III-D.2 draft pass at batch 1, and direct decoding with the parent) against
 the fp64 oracle over the same dequantised weights.
 
-The cases are shapes sq_linear_path sends to the ring (engine 3): ragged
+The cases are shapes sq_linear_path sends to the ring (engine 3), at one
+activation row and at two to eight (INT4 and FP8): ragged
 last tiles, row splits over several warps (few tiles) and whole-row jobs
 (many tiles), partial last stages, the epilogues (bias, SiLU gate,
 residual), calls chained on one stream that read the previous call's output
@@ -59,14 +60,15 @@ class _Op:
 
     def __init__(self, kind, seed, N, K, x, epi=NONE, bias=False, residual=None):
         rows = 2 * N if epi == SILU else N
-        assert sq.sq_linear_path(WK[kind], 1, N, K, epi) == 3, (kind, N, K, epi)
+        M = x.shape[0]
+        assert sq.sq_linear_path(WK[kind], M, N, K, epi) == 3, (kind, M, N, K, epi)
         self.w16 = synth.weights_fp16_device(seed, rows, K, dev())
         self.wd, self.sd = _codes(kind, self.w16, rows, K)
         self.kind, self.N, self.K, self.epi, self.x = kind, N, K, epi, x
         self.bias = f16_to_dev(synth.weights_fp16(seed + 1, 1, rows, std=0.5)[0]) if bias else None
         self.residual = residual
         self.res64 = dev_to_f64(residual) if residual is not None else None
-        self.y = torch.full((1, N), 9.0, dtype=torch.float16, device=dev())
+        self.y = torch.full((M, N), 9.0, dtype=torch.float16, device=dev())
 
     def run(self, stream=None):
         sq.sq_linear_ex(WK[self.kind], self.x, self.wd, self.sd, self.bias, self.residual, self.epi, self.y,
@@ -102,6 +104,29 @@ CASES = [
     # FP8 lm_head-like (>= 400 Mi weights)
     ("fp8", 110003, 4096, NONE), ("fp8", 51203, 8192 + 128, RES),
 ]
+
+
+# two to eight activation rows (INT4 and FP8 drafts at batch > 1): every
+# row count's column layout, ragged tiles, the K split, the epilogues
+CASES_M = [
+    ("int4", 2, 7168 + 5, 5120, NONE), ("int4", 3, 1000, 2048, RES), ("int4", 4, 13824, 5120, SILU),
+    ("int4", 5, 5120, 5120, NONE), ("int4", 8, 4133, 1536, SILU), ("int4", 8, 152064, 5120, NONE),
+    ("int4", 4, 5120, 13824, RES), ("fp8", 8, 7168, 5120, NONE), ("fp8", 5, 300, 1024, SILU),
+    ("fp8", 4, 37, 13824, RES),
+]
+
+
+@pytest.mark.parametrize("kind,M,N,K,epi", CASES_M)
+def test_ring_rows_match_oracle(kind, M, N, K, epi):
+    x = f16_to_dev(synth.activations_fp16(N % 1000 + K + M, M, K))
+    res = f16_to_dev(synth.activations_fp16(N % 777 + M, M, N)) if epi == RES else None
+    op = _Op(kind, N * 7 + K + M, N, K, x, epi=epi, bias=(N % 2 == 1), residual=res)
+    op.run()
+    assert sq.sq_check() == 0
+    op.check(f"{kind} M={M} N={N} K={K} epi={epi}", ncols=768, seed=M)
+    first = op.y.clone()
+    op.run()
+    assert torch.equal(first, op.y), "repeat not bit-identical"
 
 
 @pytest.mark.parametrize("kind,N,K,epi", CASES)

@@ -138,10 +138,10 @@ SMALL_M_TC = [
     ("fp16", 8, 200, 1000, sq.SQ_EPI_NONE),
     ("fp16", 9, 1536, 1536, sq.SQ_EPI_NONE),
     ("fp16", 15, 300, 640, sq.SQ_EPI_NONE),
-    ("fp8", 8, 200, 1024, sq.SQ_EPI_NONE),
+    ("fp8", 9, 200, 1024, sq.SQ_EPI_NONE),
     ("fp8", 9, 384, 8960, sq.SQ_EPI_NONE),
     ("fp8", 12, 256, 1536, sq.SQ_EPI_SILU_GATE),
-    ("int4", 8, 1024, 8192, sq.SQ_EPI_NONE),
+    ("int4", 9, 1024, 8192, sq.SQ_EPI_NONE),
     ("int4", 13, 2048, 4096, sq.SQ_EPI_NONE),
 ]
 
@@ -175,8 +175,10 @@ def test_engine_choice_small_rows():
     assert sq.sq_linear_path(sq.SQ_W_FP8, 1, 151936, 1536, sq.SQ_EPI_NONE) == 0
     assert sq.sq_linear_path(sq.SQ_W_FP16, 5, 2048, 1536, sq.SQ_EPI_NONE) == 0
     assert sq.sq_linear_path(sq.SQ_W_FP16, 5, 151936, 1536, sq.SQ_EPI_NONE) == 0
-    assert sq.sq_linear_path(sq.SQ_W_FP8, 5, 17920, 1536, sq.SQ_EPI_NONE) == 0
-    assert sq.sq_linear_path(sq.SQ_W_INT4, 8, 2048, 1536, sq.SQ_EPI_NONE) == 0
+    # two to eight INT4 / FP8 rows: the shared-memory ring engine
+    assert sq.sq_linear_path(sq.SQ_W_FP8, 5, 17920, 1536, sq.SQ_EPI_NONE) == 3
+    assert sq.sq_linear_path(sq.SQ_W_INT4, 8, 2048, 1536, sq.SQ_EPI_NONE) == 3
+    assert sq.sq_linear_path(sq.SQ_W_INT4, 8, 5120, 13824, sq.SQ_EPI_NONE) == 1  # 8 rows x 13824: no room
     # from 16 rows on: tensor cores
     assert sq.sq_linear_path(sq.SQ_W_INT4, 16, 2048, 1536, sq.SQ_EPI_NONE) == 1
     assert sq.sq_linear_path(sq.SQ_W_FP16, 16, 128, 64, sq.SQ_EPI_NONE) == 1
