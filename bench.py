@@ -421,6 +421,72 @@ def measure_all_configs(ctx, head_stack, reps):
     return out
 
 
+def measure_router(ctx, stack, n_prompts=24, new_tokens=32, K=4, seed=81):
+    """Sec. III-B end to end: synthetic prompt features routed by
+    router.route to INT4-draft or FP8-draft speculative decoding or direct
+    FP16 decoding; each class's sequences generate as one batch through the
+    device-side cycle (greedy), timed; compared with decoding every prompt
+    directly and with drafting every prompt with INT4.  The features are
+    synthetic (length 16..600 tokens, depth 0..10, 0..0.25 entities per
+    token); the generated prompts are 32 synthetic token ids each.  With
+    random-init weights the drafts agree with the parent almost never, so
+    the speculative classes emit about one token per cycle: the numbers
+    measure the machinery, not the paper's acceptance."""
+    import numpy as np
+
+    from paper_2609_21704_gb300 import router
+    from paper_2609_21704_gb300.generate import Generator
+
+    torch, synth, stream = ctx["torch"], ctx["synth"], ctx["stream"]
+    rng = np.random.default_rng(seed)
+    feats = [router.PromptFeatures(int(rng.integers(16, 601)), float(rng.uniform(0, 10)),
+                                   float(rng.uniform(0, 0.25))) for _ in range(n_prompts)]
+    groups = router.route_batch(feats)
+    P = 32
+    V = stack.shape.vocab
+    prompts = synth.prompt_tokens(seed + 1, n_prompts, P, V)
+    cycles = new_tokens
+
+    def gen(idx, k, draft):
+        if not idx:
+            return 0.0, 0
+        B = len(idx)
+        g = Generator(stack, B, k, P, P + 1 + k + (cycles + 2) * (k + 1), draft=draft, seed=seed + 7)
+        g.prefill(prompts[idx], stream)
+        g.run(2, stream)
+        stream.synchronize()
+        l0 = g.len.cpu().numpy().copy()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        g.run(cycles, stream)
+        e1.record(stream)
+        e1.synchronize()
+        if g.status() != 0:
+            raise RuntimeError("router generation flagged the device status word")
+        made = int((g.len.cpu().numpy() - l0).sum())
+        del g
+        return e0.elapsed_time(e1) / 1e3, made
+
+    out = {"prompts": n_prompts, "shares": {r: len(v) / n_prompts for r, v in groups.items()},
+           "thresholds": {"weights": list(router.WEIGHTS), "cuts": list(router.CUTS)}}
+    t_tot, n_tot = 0.0, 0
+    for r, idx in groups.items():
+        t, n = gen(idx, 0 if r == "fp16" else K, "int4" if r == "fp16" else r)
+        out[f"{r}_tokens_per_s"] = n / t if t else None
+        t_tot += t
+        n_tot += n
+    out["routed_tokens_per_s"] = n_tot / t_tot
+    every = list(range(n_prompts))
+    t, n = gen(every, 0, "int4")
+    out["all_direct_fp16_tokens_per_s"] = n / t
+    t, n = gen(every, K, "int4")
+    out["all_int4_draft_tokens_per_s"] = n / t
+    out["note"] = ("random-init weights: drafts almost never agree with the parent, so speculative "
+                   "classes emit ~1 token per cycle; the paper's speedups need trained weights")
+    return out
+
+
 # ----------------------------------------------------------------------------- CPU oracle leg
 
 def cpu_oracle_prepare(shape, variant, B, K, layers=1, lm_rows=None, seed=0):
@@ -818,13 +884,14 @@ def main():
         }
 
     # ---- every workload's cycle (N = 1 only: the scaling runs time the headline)
-    per_config = None
+    per_config = router_leg = None
     if world == 1 and not args.no_per_config:
         mctx = {"sq": sq, "stk": stk, "synth": synth, "torch": torch, "dev": dev, "stream": stream,
                 "capture": capture, "timed": timed, "peak": peak_gbs}
         t_pc = time.perf_counter()
         per_config = measure_all_configs(mctx, stack, reps)
         per_config["wall_s"] = round(time.perf_counter() - t_pc, 1)
+        router_leg = measure_router(mctx, stack)
     tensor_peak, tensor_peak_kind = measured_tensor_peak()
     pf_flops = 2.0 * 256 * stack.params()
     draft_bytes = stack.weight_bytes(args.draft) + stack.activation_bytes(B)
@@ -962,6 +1029,7 @@ def main():
             "decoder_speedup_vs_direct_fp16": (mean_tokens / t_dc) / (1.0 / t_ddir),
             "generation": gen,
             "per_config": per_config,
+            "router": router_leg,
             "prefill_m256_fp16_ms": 1e3 * t_pf16,
             "prefill_m256_fp16_tflops": pf_flops / t_pf16 / 1e12,
             "prefill_m256_%s_ms" % args.draft: 1e3 * t_pfd,

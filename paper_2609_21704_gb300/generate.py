@@ -37,9 +37,14 @@ ATTN_MAX_T = 32
 ATTN_MAX_GROUP_QUERIES = 200
 
 
-def prefill_chunk(q_heads: int, kv_heads: int) -> int:
-    """Tokens per prefill pass: as many as one attention call takes."""
-    return min(ATTN_MAX_T, ATTN_MAX_GROUP_QUERIES // (q_heads // kv_heads))
+# Rows of one linear call (sq_linear_ex): B sequences x T tokens of a pass.
+LINEAR_MAX_ROWS = 256
+
+
+def prefill_chunk(q_heads: int, kv_heads: int, B: int = 1) -> int:
+    """Tokens per prefill pass: as many as one attention call takes, and at
+    most LINEAR_MAX_ROWS rows over the B sequences."""
+    return max(1, min(ATTN_MAX_T, ATTN_MAX_GROUP_QUERIES // (q_heads // kv_heads), LINEAR_MAX_ROWS // B))
 
 
 class Generator:
@@ -72,7 +77,7 @@ class Generator:
             self.d2 = DecoderState(stack, B, 2, max_ctx, share_gains=self.tv)
             if K > 1:
                 self.d1 = DecoderState(stack, B, 1, max_ctx, share=self.d2)
-        pc = prefill_chunk(sh.q_heads, sh.kv_heads)
+        pc = prefill_chunk(sh.q_heads, sh.kv_heads, B)
         self.chunks = [(s, min(pc, prompt_len - s)) for s in range(0, prompt_len, pc)]
         self.pre_t, self.pre_d = {}, {}
         for _, T in self.chunks:

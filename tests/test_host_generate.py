@@ -23,3 +23,5 @@ def test_prefill_chunk_values():
     assert prefill_chunk(28, 4) == 28    # 7B: 7 per group, 7 * 32 = 224 > 200
     assert prefill_chunk(40, 8) == 32    # 14B: 5 per group
     assert prefill_chunk(200, 1) == 1
+    assert prefill_chunk(40, 8, 12) == 21   # 12 sequences: 21 x 12 = 252 rows <= 256
+    assert prefill_chunk(12, 2, 300) == 1
