@@ -32,7 +32,12 @@
 // the S partials in rank order through distributed shared memory, so the
 // result does not depend on timing.  Every mbarrier wait is bounded (a wait
 // that gives up sets SQ_DEV_TIMEOUT and is skipped from then on), so every
-// thread always reaches the cluster barriers.
+// thread always reaches the cluster barriers.  After a wait gives up, the
+// TMA producer requests nothing more and waits (bounded) for the copies it
+// still has in flight, the MMA issuer issues nothing more, and the epilogue
+// waits (bounded) on the commit that tracks every MMA issued before it
+// reads TMEM and the allocation is released; the tile's results are then
+// invalid and the status bit says so.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -247,12 +252,15 @@ __global__ void __launch_bounds__(TcConv<WK>::threads, 1)
       for (int it = 0; it < pre; ++it)
         tma_load_2d(stages + (size_t)it * a.stage_bytes + a.b_off, &tx, (k_begin + it) * kTcBK, 0,
                     &full[it]);
+      int issued = pre;  // iterations whose copies were requested
       for (int it = pre; it < nk; ++it) {
         const int s = it % a.nstages;
         const uint32_t ph = (uint32_t)(it / a.nstages) & 1u;
-        if (!timed_out && !mbar_wait_bounded(&empty[s], ph ^ 1u)) {
+        if (!mbar_wait_bounded(&empty[s], ph ^ 1u)) {
+          // the stage was never released: request nothing more
           timed_out = true;
           atomicOr(&g_tc_status, SQ_DEV_TIMEOUT);
+          break;
         }
         uint8_t* st = stages + (size_t)s * a.stage_bytes;
         const int k0 = (k_begin + it) * kTcBK;
@@ -260,6 +268,15 @@ __global__ void __launch_bounds__(TcConv<WK>::threads, 1)
         tma_load_2d(st + wdst, &tw, wx(k0), (int)(tile * kTcBM), &full[s]);
         if (SILU) tma_load_2d(st + wdst_up, &tw, wx(k0), (int)(a.N + tile * kTcBM), &full[s]);
         tma_load_2d(st + a.b_off, &tx, k0, 0, &full[s]);
+        issued = it + 1;
+      }
+      if (timed_out) {
+        // each stage has at most one request outstanding (its last): wait for
+        // it (bounded) so that no copy lands after the CTA has left
+        for (int s = 0; s < a.nstages && s < issued; ++s) {
+          const int last = s + ((issued - 1 - s) / a.nstages) * a.nstages;
+          mbar_wait_bounded(&full[s], (uint32_t)(last / a.nstages) & 1u, 1u << 20);
+        }
       }
     }
   } else if (warp == 1) {
@@ -268,9 +285,12 @@ __global__ void __launch_bounds__(TcConv<WK>::threads, 1)
       for (int it = 0; it < nk; ++it) {
         const int s = it % a.nstages;
         const uint32_t ph = (uint32_t)(it / a.nstages) & 1u;
-        if (!timed_out && !mbar_wait_bounded(QUANT ? &conv[s] : &full[s], ph)) {
+        if (!mbar_wait_bounded(QUANT ? &conv[s] : &full[s], ph)) {
+          // the stage never arrived: issue no MMA on it or after it (the
+          // commit below still tracks every MMA issued so far)
           timed_out = true;
           atomicOr(&g_tc_status, SQ_DEV_TIMEOUT);
+          break;
         }
         tc_fence_after();
         const uint32_t st = smem_u32(stages + (size_t)s * a.stage_bytes);
