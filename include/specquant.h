@@ -174,7 +174,7 @@ SQ_API sq_status sq_linear_norm(sq_wkind wkind, const void* x, const void* gamma
                                 sq_epilogue epi, void* y, int M, int64_t N, int64_t K, sq_stream_t stream);
 
 /* Engine sq_linear_ex would use for these sizes: 1 = tcgen05 tensor cores,
- * 0 = CUDA-core GEMV, 2 = one INT4 activation row over at least 304 16-row
+ * 0 = CUDA-core GEMV, 2 = one INT4 activation row over at least 192 16-row
  * output tiles with the products on the tensor cores' register-operand path
  * (mma.sync), 3 = one to eight activation rows streamed through a
  * shared-memory ring of asynchronous copies, products on the same

@@ -68,8 +68,11 @@ __device__ __forceinline__ uint32_t norm_f16x2(uint32_t xw, uint32_t gw, float r
 
 // SILU: gate rows [0, N) and up rows [N, 2N) of the weight, tile by tile;
 // S: warps sharing one tile's K range.
-template <bool SILU, int S>
-__global__ void __launch_bounds__(kMmaThreads, 4) gemv_mma_int4_kernel(const GemvArgs a) {
+// PIPE: two register batches alternate (the next batch's loads are issued
+// before the current batch's products); 80 registers, three CTAs per SM.
+// Without it, one batch at a time at 64 registers and four CTAs per SM.
+template <bool SILU, int S, bool PIPE>
+__global__ void __launch_bounds__(kMmaThreads, PIPE ? 3 : 4) gemv_mma_int4_kernel(const GemvArgs a) {
   constexpr int WR = SILU ? 2 : 1;     // weight tiles per output tile (gate, up)
   constexpr int TPC = kMmaWarps / S;   // output tiles a CTA works on at once
   constexpr int U = SILU ? 1 : 2;      // groups per load batch
@@ -150,39 +153,82 @@ __global__ void __launch_bounds__(kMmaThreads, 4) gemv_mma_int4_kernel(const Gem
   }
   __syncthreads();
 
+  // PIPE: two register batches alternate, so a warp always has a batch in
+  // flight (the first batch of the CTA's first set was issued before the
+  // wait on the previous kernel).
+  uint4 wb[PIPE ? U : 1][WR][2];
+  __half2 sb[PIPE ? U : 1][WR];
+  auto load_into = [&](uint4 (&dw)[PIPE ? U : 1][WR][2], __half2 (&ds)[PIPE ? U : 1][WR], int64_t tile,
+                       int64_t jb) {
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int64_t j = jb + u;
+#pragma unroll
+      for (int h = 0; h < WR; ++h) {
+        __half s2[2];
+#pragma unroll
+        for (int rr = 0; rr < 2; ++rr) {
+          const int64_t n = tile * 16 + g + 8 * rr;
+          const bool ok = j < j1 && tile < ntiles && n < a.N;
+          const int64_t row = (h ? a.N : 0) + (ok ? n : 0);
+          dw[u][h][rr] = ok ? ld_stream16(a.w + row * a.row_bytes + j * 64 + t * 16)
+                            : make_uint4(0u, 0u, 0u, 0u);
+          s2[rr] = ok ? gscale[row * G + j] : __ushort_as_half(0);
+        }
+        ds[u][h] = __halves2half2(s2[0], s2[1]);
+      }
+    }
+  };
+  // products of one batch (groups jb .. jb + U - 1) into acc
+  auto compute = [&](const uint4 (&cw)[U][WR][2], const __half2 (&cs)[U][WR], int64_t jb, float (&acc)[WR][2]) {
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int64_t j = jb + u;
+      if (j >= j1) break;  // warp-uniform
+      float d[WR][4];
+#pragma unroll
+      for (int h = 0; h < WR; ++h) d[h][0] = d[h][1] = d[h][2] = d[h][3] = 0.0f;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint4 xq = xm[j * 16 + t * 4 + q];
+#pragma unroll
+        for (int h = 0; h < WR; ++h) {
+          uint32_t p0[4], p1[4];  // rows g and g + 8: (k0,k4) (k1,k5) (k2,k6) (k3,k7)
+          const uint4 w0 = cw[u][h][0], w1 = cw[u][h][1];
+          int4x8_to_f16x2(q == 0 ? w0.x : q == 1 ? w0.y : q == 2 ? w0.z : w0.w, p0);
+          int4x8_to_f16x2(q == 0 ? w1.x : q == 1 ? w1.y : q == 2 ? w1.z : w1.w, p1);
+          mma_16816(d[h], p0[0], p1[0], p0[2], p1[2], xq.x, xq.y);
+          mma_16816(d[h], p0[1], p1[1], p0[3], p1[3], xq.z, xq.w);
+        }
+      }
+#pragma unroll
+      for (int h = 0; h < WR; ++h) {
+        const float2 sc = __half22float2(cs[u][h]);
+        acc[h][0] = fmaf(sc.x, d[h][0], acc[h][0]);  // row g, column 2t
+        acc[h][1] = fmaf(sc.y, d[h][2], acc[h][1]);  // row g + 8
+      }
+    }
+  };
+
   for (int64_t set = blockIdx.x; set < nsets; set += gridDim.x) {
     const int64_t tile = set * TPC + warp / S;
     float acc[WR][2];  // rows g and g + 8 of each weight tile
 #pragma unroll
     for (int h = 0; h < WR; ++h) acc[h][0] = acc[h][1] = 0.0f;
-    for (int64_t jb = j0; jb < j1; jb += U) {
-      if (set != (int64_t)blockIdx.x || jb != j0) load(tile, jb);
-#pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int64_t j = jb + u;
-        if (j >= j1) break;  // warp-uniform
-        float d[WR][4];
-#pragma unroll
-        for (int h = 0; h < WR; ++h) d[h][0] = d[h][1] = d[h][2] = d[h][3] = 0.0f;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const uint4 xq = xm[j * 16 + t * 4 + q];
-#pragma unroll
-          for (int h = 0; h < WR; ++h) {
-            uint32_t p0[4], p1[4];  // rows g and g + 8: (k0,k4) (k1,k5) (k2,k6) (k3,k7)
-            const uint4 w0 = wv[u][h][0], w1 = wv[u][h][1];
-            int4x8_to_f16x2(q == 0 ? w0.x : q == 1 ? w0.y : q == 2 ? w0.z : w0.w, p0);
-            int4x8_to_f16x2(q == 0 ? w1.x : q == 1 ? w1.y : q == 2 ? w1.z : w1.w, p1);
-            mma_16816(d[h], p0[0], p1[0], p0[2], p1[2], xq.x, xq.y);
-            mma_16816(d[h], p0[1], p1[1], p0[3], p1[3], xq.z, xq.w);
-          }
+    if constexpr (PIPE) {
+      if (set != (int64_t)blockIdx.x) load(tile, j0);
+      for (int64_t jb = j0; jb < j1; jb += 2 * U) {
+        if (jb + U < j1) load_into(wb, sb, tile, jb + U);
+        compute(wv, sv, jb, acc);
+        if (jb + U < j1) {
+          if (jb + 2 * U < j1) load_into(wv, sv, tile, jb + 2 * U);
+          compute(wb, sb, jb + U, acc);
         }
-#pragma unroll
-        for (int h = 0; h < WR; ++h) {
-          const float2 s = __half22float2(sv[u][h]);
-          acc[h][0] = fmaf(s.x, d[h][0], acc[h][0]);  // row g, column 2t
-          acc[h][1] = fmaf(s.y, d[h][2], acc[h][1]);  // row g + 8
-        }
+      }
+    } else {
+      for (int64_t jb = j0; jb < j1; jb += U) {
+        if (set != (int64_t)blockIdx.x || jb != j0) load(tile, jb);
+        compute(wv, sv, jb, acc);
       }
     }
     // ---- the S shares of K in warp order, then the epilogue (lane t == 0
@@ -222,9 +268,9 @@ __global__ void __launch_bounds__(kMmaThreads, 4) gemv_mma_int4_kernel(const Gem
 // Shared memory of one CTA: x in MMA order, then the partial sums.
 inline size_t gemv_mma_smem_bytes(int64_t K) { return (size_t)K * 2 + (size_t)kMmaWarps * 2 * 16 * 4; }
 
-template <bool SILU, int S>
+template <bool SILU, int S, bool PIPE>
 cudaError_t launch_mma_inst(const GemvArgs& a, size_t smem, cudaStream_t st) {
-  auto k = gemv_mma_int4_kernel<SILU, S>;
+  auto k = gemv_mma_int4_kernel<SILU, S, PIPE>;
   static int occ_cache[64] = {0};  // per device: resident CTAs per SM
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -256,11 +302,26 @@ inline int gemv_mma_split(int64_t N, int64_t K) {
   return S;
 }
 
+// The pipelined form when the whole grid is one wave at three CTAs per SM
+// (measured on the 14B shapes, us per launch: q/k/v 7.71 -> 7.12, o 7.31 ->
+// 6.83, down 15.54 -> 12.82; larger grids lose more to the lower occupancy
+// than they gain: lm_head 82.3 -> 90.2, the 1.5B fused gate/up 5.0 -> 6.5).
+inline bool gemv_mma_pipelined(int64_t N, int S) {
+  const int64_t tiles = (N + 15) / 16;
+  const int64_t nsets = (tiles + kMmaWarps / S - 1) / (kMmaWarps / S);
+  return nsets <= 3 * (int64_t)device_sm_count();
+}
+
 inline cudaError_t launch_gemv_mma_int4_impl(const GemvArgs& a, bool silu, cudaStream_t st) {
   const size_t smem = gemv_mma_smem_bytes(a.K);
   const int S = gemv_mma_split(a.N, a.K);
-#define SQ_MMA_CASE(S_)                                                               \
-  if (S == S_) return silu ? launch_mma_inst<true, S_>(a, smem, st) : launch_mma_inst<false, S_>(a, smem, st);
+  const bool pipe = gemv_mma_pipelined(a.N, S);
+#define SQ_MMA_CASE(S_)                                                                           \
+  if (S == S_) {                                                                                  \
+    if (pipe) return silu ? launch_mma_inst<true, S_, true>(a, smem, st)                           \
+                          : launch_mma_inst<false, S_, true>(a, smem, st);                          \
+    return silu ? launch_mma_inst<true, S_, false>(a, smem, st) : launch_mma_inst<false, S_, false>(a, smem, st); \
+  }
   SQ_MMA_CASE(1)
   SQ_MMA_CASE(2)
   SQ_MMA_CASE(4)

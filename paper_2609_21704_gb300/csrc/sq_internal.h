@@ -80,12 +80,13 @@ cudaError_t launch_gemv_fp8(const GemvArgs& a, int mr, int r, bool silu, int lpr
 cudaError_t launch_gemv_fp16(const GemvArgs& a, int mr, int r, bool silu, int lpr, int64_t blocks_needed,
                              size_t smem, cudaStream_t st);
 // INT4 weights, one activation row, products on the tensor cores' register
-// path (sq_gemv_mma.cuh); used from kMmaMinTiles 16-row output tiles on (the
-// fused gate/up and lm_head of the 1.5B/7B/14B stacks).  Measured on the
-// 1.5B draft pass: gate/up 4.99 vs 5.20 us per launch; with q/k/v, o and
-// down (96-128 tiles) on it too the pass is 576 us against 450 (too few
-// warps per SM to keep the loads in flight).
-constexpr int64_t kMmaMinTiles = 2 * kNumSMs;
+// path (sq_gemv_mma.cuh); used from kMmaMinTiles 16-row output tiles on (every
+// projection of the 7B and 14B stacks the ring engine does not take, the
+// 1.5B fused gate/up and lm_head).  Measured: 1.5B draft pass with its
+// q/k/v, o and down (96-128 tiles) on it too 170 us against 150 per 8
+// layers (too few warps per SM to keep the loads in flight); the 7B ones
+// (224-288 tiles) gain, 433 -> 403 us per 8 layers.
+constexpr int64_t kMmaMinTiles = 192;
 cudaError_t launch_gemv_mma_int4(const GemvArgs& a, bool silu, cudaStream_t st);
 inline bool gemv_uses_mma(int wkind, int M, int64_t N) {
   return wkind == SQ_W_INT4 && M == 1 && (N + 15) / 16 >= kMmaMinTiles;

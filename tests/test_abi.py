@@ -129,7 +129,7 @@ def test_single_row_engine_choice(lib):
     fused gate/up of >= 64 Mi weights, FP16 fused gate/up of >= 16 Mi and
     lm_head rows, FP8 lm_head of >= 400 Mi weights), two to eight INT4 or
     FP8 rows take it whenever their activations fit; otherwise one INT4 row
-    over at least 304 16-row output tiles takes the register-operand tensor
+    over at least 192 16-row output tiles takes the register-operand tensor
     path (2) and other few-row calls the streaming CUDA-core GEMV (0).  (The
     tcgen05 path (1) needs a device to encode its tensor maps: checked in
     tests/test_gpu_tc.py.)"""
@@ -143,9 +143,11 @@ def test_single_row_engine_choice(lib):
     assert sq.sq_linear_path(W4, 1, 2048, 1536, NONE) == 0      # 1.5B q/k/v
     assert sq.sq_linear_path(W4, 1, 1536, 1536, RES) == 0       # 1.5B o
     assert sq.sq_linear_path(W4, 1, 1536, 8960, RES) == 0       # 1.5B down
-    assert sq.sq_linear_path(W4, 1, 16 * 304, 896, NONE) == 2   # exactly 304 tiles
-    assert sq.sq_linear_path(W4, 1, 16 * 304 - 16, 896, NONE) == 0
-    assert sq.sq_linear_path(W4, 1, 16 * 303 + 1, 896, NONE) == 2  # ragged 304th tile
+    assert sq.sq_linear_path(W4, 1, 16 * 192, 896, NONE) == 2   # exactly 192 tiles
+    assert sq.sq_linear_path(W4, 1, 16 * 192 - 16, 896, NONE) == 0
+    assert sq.sq_linear_path(W4, 1, 16 * 191 + 1, 896, NONE) == 2  # ragged 192nd tile
+    assert sq.sq_linear_path(W4, 1, 4608, 3584, NONE) == 2      # 7B q/k/v (288 tiles)
+    assert sq.sq_linear_path(W4, 1, 3584, 18944, RES) == 2      # 7B down (224 tiles)
     assert sq.sq_linear_path(W4, 1, 32768, 2176, SILU) == 2     # 17 groups: odd, not the ring
     assert sq.sq_linear_path(W4, 2, 151936, 1536, NONE) == 3    # two rows: the ring too
     assert sq.sq_linear_path(W8, 8, 7168, 5120, NONE) == 3      # FP8 draft at batch 8
