@@ -7,7 +7,7 @@
 // measured faster than the GEMV family; the engine rule is in sq_plan.cu.
 //
 // Design:
-//   * one CTA per SM (16 warps for INT4, 8 for FP16 / FP8) takes a
+//   * one CTA per SM (12 or 16 warps for INT4, 8 for FP16 / FP8) takes a
 //     contiguous share of the 16-row output tiles; each warp owns a private
 //     ring of NS 4 KB slots and walks its jobs (one tile, one range of
 //     64-byte row units; a tile's units are split over S warps when tiles
@@ -40,10 +40,15 @@ namespace sq {
 
 namespace {
 
-// Warps per CTA: 8 for FP16 / FP8 (memory-bound), 16 for INT4 (bound by the
-// nibble conversion: the whole SM's warps hide its latency; 8 warps measured
-// 1.3x slower) unless the staged activations leave no room for them.
+// Warps per CTA: 8 for FP16 / FP8 (memory-bound); for INT4 (bound by the
+// nibble conversion: many warps hide its latency; 8 warps measured 1.3x
+// slower at one row) 16 at one or two activation rows and 12 from three rows
+// on, unless the staged activations leave no room for them.  Measured on the
+// 14B draft pass: 12 warps (up to 168 registers a thread instead of 128)
+// take 4 rows in 599 us against 654 us with 16 and 8 rows in 753 us against
+// 864 us, but cost 2-10 us at one and two rows; 10 or 14 warps are no better.
 constexpr int kWarpsHalf = 8;
+constexpr int kWarpsMid = 12;
 constexpr int kWarpsFull = 16;
 constexpr int kStageBytes = 4096;          // weights of one ring slot
 constexpr int kScaleBytes = 128;           // INT4 group scales of one slot
@@ -331,7 +336,7 @@ __device__ __forceinline__ void ring_store(const RingArgs& a, int64_t n, int m, 
 }
 
 template <int WK, bool SILU, int NW>
-__global__ void __launch_bounds__(NW * 32, 16 / NW) ring_linear_kernel(const RingArgs a) {
+__global__ void __launch_bounds__(NW * 32, NW > 8 ? 1 : 2) ring_linear_kernel(const RingArgs a) {
   constexpr int UPS = SILU ? kUps32 : kUps16;
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -534,12 +539,15 @@ int ring_x_stride(int M, int64_t K) {
 }
 int ring_x_bytes(int M, int64_t K) { return (M * ring_x_stride(M, K) + 127) / 128 * 128; }
 
-// Warps per CTA: 8 for FP16 / FP8; 16 for INT4 when two slots per warp fit
-// beside the staged activations, else 8.
+// Warps per CTA: 8 for FP16 / FP8; for INT4 16 (one or two rows) or 12
+// (three or more) when two slots per warp fit beside the staged activations,
+// else the next smaller count that fits.
 int ring_warps(int wkind, int M, int64_t K) {
   if (wkind != SQ_W_INT4) return kWarpsHalf;
-  return ring_smem(kWarpsFull, ring_x_bytes(M, K), 2, 4096, 128) <= (size_t)kSmemFull ? kWarpsFull
-                                                                                      : kWarpsHalf;
+  const int xb = ring_x_bytes(M, K);
+  if (M <= 2 && ring_smem(kWarpsFull, xb, 2, 4096, 128) <= (size_t)kSmemFull) return kWarpsFull;
+  if (ring_smem(kWarpsMid, xb, 2, 4096, 128) <= (size_t)kSmemFull) return kWarpsMid;
+  return kWarpsHalf;
 }
 
 template <int WK, bool SILU, int NW>
@@ -565,6 +573,9 @@ cudaError_t launch_wk(const RingArgs& a, int nw, size_t smem, int grid, cudaStre
     if (nw == kWarpsFull)
       return silu ? launch_inst<WK, true, kWarpsFull>(a, smem, grid, st)
                   : launch_inst<WK, false, kWarpsFull>(a, smem, grid, st);
+    if (nw == kWarpsMid)
+      return silu ? launch_inst<WK, true, kWarpsMid>(a, smem, grid, st)
+                  : launch_inst<WK, false, kWarpsMid>(a, smem, grid, st);
   }
   return silu ? launch_inst<WK, true, kWarpsHalf>(a, smem, grid, st)
               : launch_inst<WK, false, kWarpsHalf>(a, smem, grid, st);

@@ -113,6 +113,9 @@ CASES_M = [
     ("int4", 5, 5120, 5120, NONE), ("int4", 8, 4133, 1536, SILU), ("int4", 8, 152064, 5120, NONE),
     ("int4", 4, 5120, 13824, RES), ("fp8", 8, 7168, 5120, NONE), ("fp8", 5, 300, 1024, SILU),
     ("fp8", 4, 37, 13824, RES),
+    # INT4 warp counts when the staged rows leave less room: 12 warps at two
+    # rows of K = 27648, 8 warps at eight rows of K = 8192
+    ("int4", 2, 3000, 27648, SILU), ("int4", 8, 1000 + 3, 8192, RES),
 ]
 
 
