@@ -5,6 +5,8 @@
 #include <stdio.h>
 #include <stdlib.h>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include <cmath>
 #include <string>
 
@@ -31,6 +33,18 @@ static sq_status cuda_fail(cudaError_t e, const char* where) {
 
 static bool aligned(const void* p, uintptr_t a) { return ((uintptr_t)p % a) == 0; }
 
+// One NVTX range per entry point that launches or waits on device work,
+// named after it, so that a timeline attributes every kernel to the call
+// that issued it.  Host-only, no allocation; with no profiler attached a push
+// and a pop cost a few nanoseconds.
+struct CallRange {
+  explicit CallRange(const char* name) { nvtxRangePushA(name); }
+  ~CallRange() { nvtxRangePop(); }
+  CallRange(const CallRange&) = delete;
+  CallRange& operator=(const CallRange&) = delete;
+};
+#define SQ_RANGE() ::sq::CallRange sq_call_range_(__func__)
+
 }  // namespace sq
 
 using namespace sq;
@@ -56,6 +70,7 @@ const char* sq_status_string(sq_status s) {
 int sq_version(void) { return 100; }
 
 sq_status sq_check(sq_stream_t stream, uint32_t* device_bits) {
+  SQ_RANGE();
   cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "sq_check: stream synchronize");
   uint32_t bits = 0;
@@ -89,6 +104,7 @@ size_t sq_quantized_bytes(sq_qkind kind, int64_t N, int64_t K, size_t* scale_byt
 
 sq_status sq_quantize(const void* w16, int64_t N, int64_t K, sq_qkind kind, void* codes,
                       void* scales, sq_stream_t stream) {
+  SQ_RANGE();
   if (kind != SQ_INT4_G128 && kind != SQ_FP8_E4M3_ROW)
     return fail(SQ_ERR_INVALID_ARG, "sq_quantize: unknown kind %d", (int)kind);
   if (N < 0 || K <= 0) return fail(SQ_ERR_SHAPE, "sq_quantize: N=%lld K=%lld", (long long)N, (long long)K);
@@ -210,6 +226,7 @@ static sq_status run_linear(const sq_linear_op& op, cudaStream_t stream, const _
 sq_status sq_linear_norm(sq_wkind wkind, const void* x, const void* gamma, float eps, void* xn, const void* w,
                          const void* scales, const void* bias, const void* residual, sq_epilogue epi, void* y,
                          int M, int64_t N, int64_t K, sq_stream_t stream) {
+  SQ_RANGE();
   sq_linear_op op = {};
   op.wkind = wkind;
   op.epi = epi;
@@ -238,6 +255,7 @@ sq_status sq_linear_norm(sq_wkind wkind, const void* x, const void* gamma, float
 sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void* scales,
                        const void* bias, const void* residual, sq_epilogue epi, void* y, int M,
                        int64_t N, int64_t K, sq_stream_t stream) {
+  SQ_RANGE();
   sq_linear_op op = {};
   op.wkind = wkind;
   op.epi = epi;
@@ -256,6 +274,7 @@ sq_status sq_linear_ex(sq_wkind wkind, const void* x, const void* w, const void*
 }
 
 sq_status sq_linear_chain(const sq_linear_op* ops, int count, sq_stream_t stream) {
+  SQ_RANGE();
   if (count < 0 || (count > 0 && !ops))
     return fail(SQ_ERR_INVALID_ARG, "sq_linear_chain: need ops and count >= 0");
   for (int i = 0; i < count; ++i) {
@@ -270,6 +289,7 @@ sq_status sq_linear_chain(const sq_linear_op* ops, int count, sq_stream_t stream
 }
 
 sq_status sq_selftest_wait(int which, uint64_t limit, sq_stream_t stream) {
+  SQ_RANGE();
   if (which != 0 && which != 1) return fail(SQ_ERR_INVALID_ARG, "sq_selftest_wait: which must be 0 or 1");
   if (which == 0 && (limit < 1 || limit > ((uint64_t)1 << 24)))
     return fail(SQ_ERR_INVALID_ARG, "sq_selftest_wait: polls must be in [1, 2^24]");
@@ -290,16 +310,19 @@ int sq_linear_path(sq_wkind wkind, int M, int64_t N, int64_t K, sq_epilogue epi)
 
 sq_status sq_linear_w4a16(const void* x, const void* codes, const void* scales, const void* bias,
                           void* y, int M, int64_t N, int64_t K, sq_stream_t stream) {
+  SQ_RANGE();
   return sq_linear_ex(SQ_W_INT4, x, codes, scales, bias, nullptr, SQ_EPI_NONE, y, M, N, K, stream);
 }
 
 sq_status sq_linear_fp8(const void* x, const void* codes, const float* scales, const void* bias,
                         void* y, int M, int64_t N, int64_t K, sq_stream_t stream) {
+  SQ_RANGE();
   return sq_linear_ex(SQ_W_FP8, x, codes, scales, bias, nullptr, SQ_EPI_NONE, y, M, N, K, stream);
 }
 
 sq_status sq_verify(const void* x, const void* w16, const void* bias, void* y, int M, int64_t N,
                     int64_t K, sq_stream_t stream) {
+  SQ_RANGE();
   return sq_linear_ex(SQ_W_FP16, x, w16, nullptr, bias, nullptr, SQ_EPI_NONE, y, M, N, K, stream);
 }
 
@@ -361,6 +384,7 @@ static sq_status accept_common(const char* who, const float* p, const float* q, 
 sq_status sq_accept(const float* p, const float* q, const int32_t* draft, const float* u, int B, int K,
                     int64_t V, sq_accept_mode mode, int32_t* n_accepted, int32_t* tokens,
                     void* workspace, size_t ws_bytes, sq_stream_t stream) {
+  SQ_RANGE();
   if (!n_accepted && B > 0) return fail(SQ_ERR_INVALID_ARG, "sq_accept: NULL n_accepted");
   return accept_common("sq_accept", p, q, draft, u, B, K, V, (int)mode, n_accepted, tokens, workspace,
                        ws_bytes, stream);
@@ -368,6 +392,7 @@ sq_status sq_accept(const float* p, const float* q, const int32_t* draft, const 
 
 sq_status sq_sample(const float* probs, const float* u, int B, int64_t V, int32_t* tokens,
                     void* workspace, size_t ws_bytes, sq_stream_t stream) {
+  SQ_RANGE();
   return accept_common("sq_sample", probs, nullptr, nullptr, u, B, 0, V, SQ_ACCEPT_SAMPLE, nullptr,
                        tokens, workspace, ws_bytes, stream);
 }
@@ -436,6 +461,7 @@ sq_status sq_accept_logits(const void* zp, const void* zq, const int32_t* draft,
                            int K, int64_t V, float temperature, sq_accept_mode mode,
                            int32_t* n_accepted, int32_t* tokens, void* workspace, size_t ws_bytes,
                            sq_stream_t stream) {
+  SQ_RANGE();
   if (!n_accepted && B > 0) return fail(SQ_ERR_INVALID_ARG, "sq_accept_logits: NULL n_accepted");
   return accept_logits_common("sq_accept_logits", zp, zq, draft, u, B, K, V, temperature, (int)mode,
                               n_accepted, tokens, workspace, ws_bytes, stream);
@@ -443,6 +469,7 @@ sq_status sq_accept_logits(const void* zp, const void* zq, const int32_t* draft,
 
 sq_status sq_sample_logits(const void* z, const float* u, int B, int64_t V, float temperature,
                            int32_t* tokens, void* workspace, size_t ws_bytes, sq_stream_t stream) {
+  SQ_RANGE();
   return accept_logits_common("sq_sample_logits", z, nullptr, nullptr, u, B, 0, V, temperature,
                               SQ_ACCEPT_SAMPLE, nullptr, tokens, workspace, ws_bytes, stream);
 }
@@ -451,6 +478,7 @@ size_t sq_softmax_workspace_bytes(int64_t R, int64_t V) { return softmax_rows_wo
 
 sq_status sq_softmax(const void* z, int64_t R, int64_t V, float temperature, float* p, void* workspace,
                      size_t ws_bytes, sq_stream_t stream) {
+  SQ_RANGE();
   if (R < 0 || V < 1 || V >= ((int64_t)1 << 20))
     return fail(SQ_ERR_SHAPE, "sq_softmax: need R >= 0, 1 <= V < 2^20 (R=%lld V=%lld)", (long long)R,
                 (long long)V);
@@ -481,6 +509,7 @@ sq_status sq_softmax(const void* z, int64_t R, int64_t V, float temperature, flo
 
 sq_status sq_rmsnorm(const void* x, const void* gamma, int M, int64_t H, float eps, void* y,
                      sq_stream_t stream) {
+  SQ_RANGE();
   if (M < 0 || H < 1) return fail(SQ_ERR_SHAPE, "sq_rmsnorm: need M >= 0, H >= 1");
   if (!(eps >= 0.0f) || !std::isfinite(eps)) return fail(SQ_ERR_INVALID_ARG, "sq_rmsnorm: bad eps");
   if (M == 0) return SQ_OK;
@@ -511,6 +540,7 @@ static sq_status check_attn(const char* who, const void* qkv, int B, int T, int 
 
 sq_status sq_kv_append(const void* qkv, int B, int T, int Hq, int Hkv, int D, const int32_t* pos0,
                        float theta, void* k_cache, void* v_cache, int64_t max_ctx, sq_stream_t stream) {
+  SQ_RANGE();
   sq_status st = check_attn("sq_kv_append", qkv, B, T, Hq, Hkv, D, pos0, theta, k_cache, v_cache, max_ctx);
   if (st != SQ_OK) return st;
   cudaError_t e = launch_kv_append(reinterpret_cast<const __half*>(qkv), B, T, Hq, Hkv, pos0, (double)theta,
@@ -553,6 +583,7 @@ static sq_status attention_common(const char* who, const void* qkv, int B, int T
 sq_status sq_attention(const void* qkv, int B, int T, int Hq, int Hkv, int D, const int32_t* pos0,
                        float theta, const void* k_cache, const void* v_cache, int64_t max_ctx, void* out,
                        void* workspace, size_t ws_bytes, sq_stream_t stream) {
+  SQ_RANGE();
   return attention_common("sq_attention", qkv, B, T, Hq, Hkv, D, pos0, theta, k_cache, v_cache, max_ctx, out,
                           workspace, ws_bytes, false, stream);
 }
@@ -560,12 +591,14 @@ sq_status sq_attention(const void* qkv, int B, int T, int Hq, int Hkv, int D, co
 sq_status sq_attention_append(const void* qkv, int B, int T, int Hq, int Hkv, int D, const int32_t* pos0,
                               float theta, void* k_cache, void* v_cache, int64_t max_ctx, void* out,
                               void* workspace, size_t ws_bytes, sq_stream_t stream) {
+  SQ_RANGE();
   return attention_common("sq_attention_append", qkv, B, T, Hq, Hkv, D, pos0, theta, k_cache, v_cache,
                           max_ctx, out, workspace, ws_bytes, true, stream);
 }
 
 sq_status sq_kv_rollback(const int32_t* base, const int32_t* n_accepted, int B, int limit, int32_t* len,
                          sq_stream_t stream) {
+  SQ_RANGE();
   if (B < 0 || limit < 0) return fail(SQ_ERR_SHAPE, "sq_kv_rollback: need B >= 0, limit >= 0");
   if (B == 0) return SQ_OK;
   if (!base || !n_accepted || !len) return fail(SQ_ERR_INVALID_ARG, "sq_kv_rollback: NULL pointer");
@@ -578,6 +611,7 @@ sq_status sq_kv_rollback(const int32_t* base, const int32_t* n_accepted, int B, 
 
 sq_status sq_embed(const int32_t* ids, int M, int64_t ids_stride, const void* table, int64_t V, int64_t H,
                    void* out, sq_stream_t stream) {
+  SQ_RANGE();
   if (M < 0 || V < 1 || H < 1 || ids_stride < 1)
     return fail(SQ_ERR_SHAPE, "sq_embed: need M >= 0, V >= 1, H >= 1, ids_stride >= 1");
   if (M == 0) return SQ_OK;
@@ -592,6 +626,7 @@ sq_status sq_embed(const int32_t* ids, int M, int64_t ids_stride, const void* ta
 
 sq_status sq_spec_commit(const int32_t* n_accepted, const int32_t* tokens, int ldt, int B, int K, int32_t* hist,
                          int cap, int32_t* len, int32_t* pos, int32_t* last2, sq_stream_t stream) {
+  SQ_RANGE();
   if (B < 0 || K < 0 || ldt < 1 || cap < 1)
     return fail(SQ_ERR_SHAPE, "sq_spec_commit: need B >= 0, K >= 0, ldt >= 1, cap >= 1");
   if (B == 0) return SQ_OK;
@@ -607,6 +642,7 @@ sq_status sq_spec_commit(const int32_t* n_accepted, const int32_t* tokens, int l
 
 sq_status sq_spec_drafts(const int32_t* samples, const int32_t* last2, int B, int K, int32_t* verify_tokens,
                          int32_t* draft, sq_stream_t stream) {
+  SQ_RANGE();
   if (B < 0 || K < 0) return fail(SQ_ERR_SHAPE, "sq_spec_drafts: need B >= 0, K >= 0");
   if (B == 0) return SQ_OK;
   if (!last2 || !verify_tokens || (K > 0 && (!samples || !draft)))
@@ -625,6 +661,7 @@ sq_status sq_spec_drafts(const int32_t* samples, const int32_t* last2, int B, in
 sq_status sq_accept_noalloc(const float* p, const float* q, const int32_t* draft, const float* u,
                             int B, int K, int64_t V, sq_accept_mode mode, int32_t* n_accepted,
                             int32_t* tokens, sq_stream_t stream) {
+  SQ_RANGE();
   if (B < 0 || K < 0 || K > 16 || V < 1 || V >= ((int64_t)1 << 20))
     return fail(SQ_ERR_SHAPE, "sq_accept_noalloc: need B >= 0, 0 <= K <= 16, 1 <= V < 2^20 (B=%d K=%d V=%lld)",
                 B, K, (long long)V);
