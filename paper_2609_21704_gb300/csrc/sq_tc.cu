@@ -468,9 +468,11 @@ __global__ void __launch_bounds__(TcConv<WK>::threads, 1)
     cluster_sync();  // every partial tile is written
     if (warp >= 2) {
       const int et = tid - 64;  // 0 .. blockDim.x - 65
-      const int rows = (kTcBM + S - 1) / S;  // this rank's rows [r0, r0 + nr)
+      // this rank's rows [r0, r0 + nr): shares rounded up to four rows so
+      // that every split's ranks start on a 16-byte boundary
+      const int rows = ((kTcBM + S - 1) / S + 3) & ~3;
       const int r0 = (int)rank * rows;
-      const int nr = rows < kTcBM - r0 ? rows : kTcBM - r0;
+      const int nr = max(0, min(rows, kTcBM - r0));
       const float* part = reinterpret_cast<const float*>(stages);
       const int nthr = (int)blockDim.x - 64;
       // output (column m, row) from the summed partials g (and u, the up row's)
@@ -673,7 +675,7 @@ static int tc_max_clusters(int S, size_t smem) {
 // the smaller S.
 template <int WK, bool SILU>
 static int tc_pick_split(int64_t tiles, int ksteps, size_t smem, int max_split, bool two_per_sm,
-                         bool int4_large = false) {
+                         bool int4_large = false, bool many_rows = false) {
   if (WK == 1 && int4_large) {
     // two CTAs per SM: the largest power-of-two split with at most 2.2 CTAs
     // per SM in all and at least 12 k-steps per CTA (odd splits of 3 and 7
@@ -695,6 +697,13 @@ static int tc_pick_split(int64_t tiles, int ksteps, size_t smem, int max_split, 
       return S;
     }
     // one CTA per SM: clusters of at most the portable 8 SMs
+    if (many_rows) {
+      // many activation rows (NB > 64: every k-step also streams a large
+      // activation tile and runs a long MMA): the largest S that still fits
+      // one wave
+      while (S + 1 <= max_split && S + 1 <= 8 && tiles * (S + 1) <= sms && ksteps >= 4 * (S + 1)) ++S;
+      return S;
+    }
     while (2 * S <= max_split && 2 * S <= 8 && tiles * S * 2 <= sms && ksteps >= 4 * S * 2) S <<= 1;
     return S;
   }
@@ -720,7 +729,7 @@ static cudaError_t tc_launch_inst(const CUtensorMap& tw, const CUtensorMap& tx, 
   cudaError_t e = tc_prepare<WK, SILU>(smem);
   if (e != cudaSuccess) return e;
   const int S = tc_pick_split<WK, SILU>(tiles, a.ksteps, smem, a.max_split, a.two_per_sm != 0,
-                                       a.int4_large != 0);
+                                       a.int4_large != 0, a.NB > 64);
   a.splits = S;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)S, (unsigned)tiles, 1);
