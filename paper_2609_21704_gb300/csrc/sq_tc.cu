@@ -468,13 +468,26 @@ __global__ void __launch_bounds__(TcConv<WK>::threads, 1)
     cluster_sync();  // every partial tile is written
     if (warp >= 2) {
       const int et = tid - 64;  // 0 .. blockDim.x - 65
-      // this rank's rows [r0, r0 + nr): shares rounded up to four rows so
-      // that every split's ranks start on a 16-byte boundary
-      const int rows = ((kTcBM + S - 1) / S + 3) & ~3;
+      // this rank's rows [r0, r0 + nr).  Small splits over many columns:
+      // four consecutive rows per 16-byte load of each partial and four such
+      // items in flight per thread, the shares rounded up to four rows so
+      // that every rank starts on a 16-byte boundary (14B FP16 at 144 rows,
+      // S = 2-3: qkv 42 -> 30 us, down 65 -> 53 us; the element loop there
+      // waited one cluster-load latency per element).  Otherwise one element
+      // per thread, with all S loads of an element in flight, and shares as
+      // even as possible (7B FP16 at 48 rows, S = 7-10: the four-row form,
+      // which waits one latency per rank, measured 1123 us against 1045 us
+      // per pass; INT4 at 16 rows, S = 8).  The decision depends only on S,
+      // M and the block, so every rank takes the same.  The partials are
+      // added in rank order either way.
+      const int nthr = (int)blockDim.x - 64;
+      const int rows1 = (kTcBM + S - 1) / S;
+      const int rows4 = (rows1 + 3) & ~3;
+      const bool vec = S <= 4 && (rows4 >> 2) * a.M >= nthr;
+      const int rows = vec ? rows4 : rows1;
       const int r0 = (int)rank * rows;
       const int nr = max(0, min(rows, kTcBM - r0));
       const float* part = reinterpret_cast<const float*>(stages);
-      const int nthr = (int)blockDim.x - 64;
       // output (column m, row) from the summed partials g (and u, the up row's)
       auto emit = [&](int m, int row, float g, float u) {
         const int64_t n = tile * kTcBM + row;
@@ -490,13 +503,7 @@ __global__ void __launch_bounds__(TcConv<WK>::threads, 1)
         if (a.residual) v += __half2float(a.residual[(int64_t)m * a.N + n]);
         a.y[(int64_t)m * a.N + n] = __float2half_rn(v);
       };
-      if ((r0 & 3) == 0 && (nr & 3) == 0 && (nr >> 2) * a.M >= nthr) {
-        // many columns: four consecutive rows per 16-byte load of each
-        // partial and four such items in flight per thread (the loads'
-        // latency dominates; 14B FP16 at 144 rows: qkv 42 -> 30 us, down 65
-        // -> 53 us); with fewer items than threads one element per thread
-        // keeps every warp busy (INT4 at 16 rows, S = 8).  The partials are
-        // added in rank order either way.
+      if (vec) {
         constexpr int kIt = 4;
         const int nq = nr >> 2;
         const int items = nq * a.M;
