@@ -128,9 +128,10 @@ SQ_API sq_status sq_quantize(const void* w16, int64_t N, int64_t K, sq_qkind kin
  * from (format, M, N, K, epilogue) alone (sq_linear_path reports which):
  * the CUDA-core GEMV family for few rows (for one INT4 row over many output
  * rows, with its products on the tensor cores' register-operand path), the
- * tcgen05 tensor-core tile path from 16 rows on and, below that, for the
- * formats and shapes where it is faster.  All give the same fp32-accumulated
- * result up to summation order.
+ * shared-memory ring engine for one to eight rows of large or quantised
+ * weights, and the tcgen05 tensor-core tile path from 16 rows on and, below
+ * that, for the formats and shapes where it is faster.  All give the same
+ * fp32-accumulated result up to summation order.
  * y must not overlap x, the weights or the scales.
  * ---------------------------------------------------------------------- */
 SQ_API sq_status sq_linear_w4a16(const void* x, const void* codes, const void* scales,

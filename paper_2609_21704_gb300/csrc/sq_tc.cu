@@ -28,9 +28,9 @@
 //
 // Split-K: the S CTAs of a cluster take consecutive K ranges of the same
 // weight tile; each writes its fp32 partial tile to its own shared memory,
-// and after a cluster barrier CTA r sums rows [r*128/S, (r+1)*128/S) over
-// the S partials in rank order through distributed shared memory, so the
-// result does not depend on timing.  Every mbarrier wait is bounded (a wait
+// and after a cluster barrier CTA r sums its share of the 128 rows (about
+// 128/S consecutive rows) over the S partials in rank order through
+// distributed shared memory, so the result does not depend on timing.  Every mbarrier wait is bounded (a wait
 // that gives up sets SQ_DEV_TIMEOUT and is skipped from then on), so every
 // thread always reaches the cluster barriers.  After a wait gives up, the
 // TMA producer requests nothing more and waits (bounded) for the copies it
