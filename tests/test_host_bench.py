@@ -34,3 +34,17 @@ def test_row_slices_partition_and_reproduce_the_outputs(n, silu, P):
     got = np.concatenate([_outputs(p) for p in parts if p[0] > 0], axis=1)
     assert got.shape[1] == half
     np.testing.assert_array_equal(got, _outputs(it))
+
+
+def test_workload_name_names_the_stack_and_the_cycle():
+    """Both arms name their workload with bench.workload_name: the stack,
+    its linear weight count, the draft and verify rows of one cycle and the
+    vocabulary the accept runs over."""
+    from paper_2609_21704_gb300.shapes import QWEN25_14B, QWEN25_7B
+
+    assert bench.workload_name(QWEN25_14B, "int4", 1, 4) == (
+        "qwen2.5-14b linear stack (48 layers + lm_head, 13.991B linear weights), INT4 draft "
+        "B=1 x K=4 (M=1), FP16 verify M=5, accept V=152064")
+    name = bench.workload_name(QWEN25_7B, "fp8", 8, 5)
+    assert "FP8 draft B=8 x K=5 (M=8)" in name and "FP16 verify M=48" in name
+    assert f"{QWEN25_7B.linear_params() / 1e9:.3f}B" in name
